@@ -1,0 +1,378 @@
+"""Throughput of LAST's edge-side token-selection path on GB300.
+
+One step = one pass of the whole path over one batch: last-query-token
+scores (Eq. 6-8), greedy k-center selection (Eq. 9-11) and the ordered gather
+(Eq. 12), through the C ABI (last_scores, then last_select with the fused
+gather), with the inputs already resident in device memory.
+
+Default workload: 64 requests of LLaVA-1.5 shape (576 visual tokens + 16..128
+text tokens, 16 q/kv heads x 128, bf16, 2048-d features, 64-cluster mixture),
+budgets 64 / 128 / 192 assigned round-robin over the batch.  Inputs are 321 MB,
+larger than the 129 MB L2, so no flush is needed between steps.
+
+Prints one JSON line (rank 0).  `--impl reference` times the plain C oracle
+(as it stands) on the host cores instead.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "pruned requests/sec and visual tokens scored/sec per GB300; % of HBM roofline"
+UNIT = "requests/s"
+PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
+FALLBACK_HBM_GBS = 6800.0
+SM_COUNT_NOMINAL = 152
+FP32_LANES_PER_SM = 128
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--budget", default="mixed", help="c2 budget: mixed, 64, 128 or 192")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    return ap.parse_args()
+
+
+def workload(budget, rank):
+    from workloads import config
+    b = budget if budget == "mixed" else int(budget)
+    # each rank prunes its own batch (independent requests, weak scaling)
+    return config("c2", budget=b, seed=1 + 1000 * rank)
+
+
+def workload_desc(wl, budget):
+    n = np.diff(wl.cu_vis)
+    k = np.diff(wl.cu_keep)
+    return {"workload": f"c2: {wl.batch} requests x {int(n[0])} visual tokens (LLaVA-1.5 shape), "
+                        f"budgets {'64/128/192 round-robin' if budget == 'mixed' else budget}",
+            "batch": wl.batch, "visual_tokens": int(n.sum()), "kept_tokens": int(k.sum()),
+            "keys": int(wl.cu_seqlens[-1]), "layers": wl.num_layers, "q_heads": wl.num_q_heads,
+            "kv_heads": wl.num_kv_heads, "head_dim": wl.head_dim, "feat_dim": wl.feat_dim,
+            "input_bytes": int(wl.q.nbytes + wl.k.nbytes + wl.x.nbytes),
+            "l2": "inputs (321 MB) larger than L2 (129 MB); no flush"}
+
+
+def select_fmas(wl):
+    """Algorithmic work of the selection kernel: N_b norm dots plus, at greedy step t,
+    one dot per still-unselected token (Eq. 10), each d_v FMAs."""
+    tot = 0
+    for b in range(wl.batch):
+        n = int(wl.cu_vis[b + 1] - wl.cu_vis[b])
+        k = int(wl.cu_keep[b + 1] - wl.cu_keep[b])
+        if 0 < k < n:
+            tot += n + (k - 1) * n - k * (k - 1) // 2
+    return tot * wl.feat_dim
+
+
+def score_bytes(wl):
+    """Compulsory bytes of the scoring kernels: every key once, q once, w written."""
+    return wl.k.nbytes + wl.q.nbytes + 4 * int(wl.cu_vis[-1])
+
+
+class ClockSampler:
+    """nvidia-smi clocks/throttle reasons sampled every 200 ms while running."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        if self.proc is None or not self.path or not os.path.exists(self.path):
+            return None
+        rows = []
+        for line in open(self.path):
+            p = [s.strip() for s in line.split(",")]
+            if len(p) < 9:
+                continue
+            try:
+                rows.append(dict(sm=float(p[1]), smax=float(p[2]), power=float(p[3]),
+                                 hw=p[5], hwt=p[6], swt=p[7], pcap=p[8]))
+            except ValueError:
+                continue
+        os.unlink(self.path)
+        if not rows:
+            return None
+        reasons = set()
+        for r in rows:
+            for key, name in (("hw", "hw_slowdown"), ("hwt", "hw_thermal_slowdown"),
+                              ("swt", "sw_thermal_slowdown"), ("pcap", "sw_power_cap")):
+                if r[key].lower() == "active":
+                    reasons.add(name)
+        loaded = [r for r in rows if r["power"] > 0.25 * max(x["power"] for x in rows)] or rows
+        return {"sm_mhz": statistics.median(r["sm"] for r in loaded),
+                "sm_max_mhz": max(r["smax"] for r in rows), "reasons": sorted(reasons),
+                "samples": len(rows), "power_w_max": max(r["power"] for r in rows)}
+
+
+def peaks():
+    try:
+        with open(PEAKS_FILE) as f:
+            return json.load(f), "measured"
+    except (OSError, ValueError):
+        return {"hbm_gbs": FALLBACK_HBM_GBS, "sm_max_mhz": 2070.0}, "fallback"
+
+
+def cpu_baseline(wl, budget_s=15.0):
+    """The oracle as it stands (single thread) on a bounded sample of the same batch:
+    whole requests (fp64 scores of the request, canonical-fp32 greedy, gather)."""
+    import oracle
+    from workloads import custom  # noqa: F401  (same generator as the GPU leg)
+    oracle.build()
+    t0 = time.perf_counter()
+    done = 0
+    order = [0, 1, 2] * (wl.batch // 3)
+    for b in order:
+        v0, v1 = int(wl.cu_vis[b]), int(wl.cu_vis[b + 1])
+        s0, s1 = int(wl.cu_seqlens[b]), int(wl.cu_seqlens[b + 1])
+        kb = int(wl.cu_keep[b + 1] - wl.cu_keep[b])
+        w = oracle.scores(wl.q[b:b + 1], np.ascontiguousarray(wl.k[:, s0:s1]), [0, s1 - s0],
+                          [int(wl.vis_start[b])], [0, v1 - v0], num_kv_heads=wl.num_kv_heads)
+        oracle.prune_request(wl.x[v0:v1], w.astype(np.float32), kb)
+        done += 1
+        if time.perf_counter() - t0 > budget_s:
+            break
+    dt = time.perf_counter() - t0
+    return {"value": done / dt, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"{done} whole requests of the same batch (k=64/128/192 in turn), "
+                      f"single-threaded C oracle, {dt:.1f} s"}
+
+
+def run_reference(args, rank, world):
+    """--impl reference: the oracle, as it stands, on the host cores (rank 0 only)."""
+    if rank != 0:
+        return
+    wl = workload(args.budget, 0)
+    import oracle
+    oracle.build()
+
+    def step(i):
+        # a bounded sample per step: one whole request, budgets in turn
+        b = i % 3
+        v0, v1 = int(wl.cu_vis[b]), int(wl.cu_vis[b + 1])
+        s0, s1 = int(wl.cu_seqlens[b]), int(wl.cu_seqlens[b + 1])
+        kb = int(wl.cu_keep[b + 1] - wl.cu_keep[b])
+        w = oracle.scores(wl.q[b:b + 1], np.ascontiguousarray(wl.k[:, s0:s1]), [0, s1 - s0],
+                          [int(wl.vis_start[b])], [0, v1 - v0], num_kv_heads=wl.num_kv_heads)
+        oracle.prune_request(wl.x[v0:v1], w.astype(np.float32), kb)
+        return v1 - v0
+
+    for i in range(args.warmup):
+        step(i)
+    t0 = time.perf_counter()
+    toks = 0
+    for i in range(args.steps):
+        toks += step(i)
+    dt = time.perf_counter() - t0
+    value = args.steps / dt
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1000 * dt / args.steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64 scores / f32 selection", "data": "synthetic",
+            "config": workload_desc(wl, args.budget) | {"per_step": "1 whole request (oracle)"},
+            "visual_tokens_scored_per_s": toks / dt,
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                             "sample": "1 whole request of the c2 batch per step, budgets in turn"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse()
+    rank = int(os.environ.get("RANK", 0))
+    world = int(os.environ.get("WORLD_SIZE", 1))
+    local = int(os.environ.get("LOCAL_RANK", 0))
+    if args.impl == "reference":
+        run_reference(args, rank, world)
+        return
+
+    import torch
+    import paper_2607_27952_gb300 as last
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    last.load_library()
+
+    wl = workload(args.budget, rank)
+    prob = last.Problem(batch=wl.batch, num_layers=wl.num_layers, num_q_heads=wl.num_q_heads,
+                        num_kv_heads=wl.num_kv_heads, head_dim=wl.head_dim, feat_dim=wl.feat_dim,
+                        dtype=wl.dtype, cu_seqlens=wl.cu_seqlens, vis_start=wl.vis_start,
+                        cu_vis=wl.cu_vis, cu_keep=wl.cu_keep)
+
+    def dev_t(a):
+        return torch.from_numpy(a.view(np.int16)).to(dev).view(torch.bfloat16)
+
+    q, k, x = dev_t(wl.q), dev_t(wl.k), dev_t(wl.x)
+    nvis, nkeep = int(wl.cu_vis[-1]), int(wl.cu_keep[-1])
+    w = torch.empty(nvis, dtype=torch.float32, device=dev)
+    idx = torch.empty(nkeep, dtype=torch.int32, device=dev)
+    xs = torch.empty((nkeep, wl.feat_dim), dtype=torch.bfloat16, device=dev)
+    ws = last.workspace(prob, dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def step():
+        last.last_scores(prob, q, k, w, ws, stream)
+        last.last_select(prob, w, x, idx, ws, stream, x_out=xs)
+
+    for _ in range(args.warmup):
+        step()
+    last.last_poll(ws, stream)
+
+    def barrier():
+        if world > 1:
+            torch.distributed.barrier()
+
+    K = args.steps
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(K)]
+    with ClockSampler(local) as clk:
+        barrier()
+        torch.cuda.synchronize(dev)
+        for i in range(K):
+            ev[i][0].record(stream)
+            last.last_scores(prob, q, k, w, ws, stream)
+            ev[i][1].record(stream)
+            last.last_select(prob, w, x, idx, ws, stream, x_out=xs)
+            ev[i][2].record(stream)
+        torch.cuda.synchronize(dev)
+        barrier()
+    clocks = clk.summary()
+    last.last_poll(ws, stream)
+    total_ms = ev[0][0].elapsed_time(ev[-1][2])
+    scores_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in ev)
+    select_ms = statistics.mean(e[1].elapsed_time(e[2]) for e in ev)
+    if world > 1:
+        t = torch.tensor([total_ms], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        total_ms = float(t.item())
+
+    reqs = wl.batch * world * K
+    value = reqs / (total_ms / 1e3)
+    tokens_per_s = nvis * world * K / (total_ms / 1e3)
+
+    pk, pk_kind = peaks()
+    sm_count = torch.cuda.get_device_properties(dev).multi_processor_count
+    sm_max = float(pk.get("sm_max_mhz", 2070.0))
+    alu_peak_tflops = sm_count * FP32_LANES_PER_SM * 2 * sm_max * 1e6 / 1e12
+    sel_flops = 2.0 * select_fmas(wl)
+    achieved = sel_flops / (select_ms / 1e3) / 1e12
+    hbm = float(pk.get("hbm_gbs", FALLBACK_HBM_GBS))
+    sc_gbs = score_bytes(wl) / (scores_ms / 1e3) / 1e9
+
+    e2e = None
+    if not args.no_e2e:
+        e2e = measure_e2e(args, wl, prob, dev, stream, last, q, k, x)
+
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
+        "warmup": args.warmup, "ms_per_step": total_ms / K, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16 in, fp32 compute",
+        "data": "synthetic (seeded; shapes of the paper's LLaVA-1.5 workload)",
+        "config": workload_desc(wl, args.budget) | {"parallelism": f"replicas x{world}"},
+        "visual_tokens_scored_per_s": tokens_per_s,
+        "gpu_launches": 3 * K,
+        "kernels": {"scores_ms": scores_ms, "select_ms": select_ms,
+                    "scores_GBps": sc_gbs, "scores_hbm_frac": sc_gbs / hbm},
+        "roofline": {"bound": "alu", "kernel": "select_kernel", "achieved": achieved,
+                     "peak": alu_peak_tflops, "unit": "TFLOP/s", "frac": achieved / alu_peak_tflops,
+                     "traffic": None,
+                     "peak_note": f"{sm_count} SMs x {FP32_LANES_PER_SM} fp32 FMA/clk x 2 x "
+                                  f"{sm_max:.0f} MHz ({pk_kind} max clock)"},
+        "clocks": clocks,
+    }
+    if e2e is not None:
+        line["e2e"] = e2e
+    if rank == 0 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(wl)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+def measure_e2e(args, wl, prob, dev, stream, last, q_d, k_d, x_d):
+    """The same metric through the user call last_prune with host buffers: each step
+    copies q, K, X from pinned host memory, prunes, and reads back the kept indices and
+    rows."""
+    import torch
+    pin = lambda a: torch.from_numpy(a.view(np.int16)).view(torch.bfloat16).pin_memory()
+    qh, kh, xh = pin(wl.q), pin(wl.k), pin(wl.x)
+    nkeep = int(wl.cu_keep[-1])
+    idx_h = torch.empty(nkeep, dtype=torch.int32).pin_memory()
+    xs_h = torch.empty((nkeep, wl.feat_dim), dtype=torch.bfloat16).pin_memory()
+    idx_d = torch.empty(nkeep, dtype=torch.int32, device=dev)
+    xs_d = torch.empty((nkeep, wl.feat_dim), dtype=torch.bfloat16, device=dev)
+    ws = last.workspace(prob, dev)
+
+    def step():
+        q_d.copy_(qh, non_blocking=True)
+        k_d.copy_(kh, non_blocking=True)
+        x_d.copy_(xh, non_blocking=True)
+        last.last_prune(prob, q_d, k_d, x_d, None, idx_d, xs_d, ws, stream)
+        idx_h.copy_(idx_d, non_blocking=True)
+        xs_h.copy_(xs_d, non_blocking=True)
+
+    for _ in range(max(1, args.warmup // 2)):
+        step()
+    torch.cuda.synchronize(dev)
+    steps = max(3, args.steps // 2)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    ms = e0.elapsed_time(e1)
+    h2d = int(qh.numel() + kh.numel() + xh.numel()) * 2
+    d2h = int(idx_h.numel() * 4 + xs_h.numel() * 2)
+    return {"value": wl.batch * steps / (ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h, "steps": steps}
+
+
+if __name__ == "__main__":
+    main()

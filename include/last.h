@@ -1,0 +1,143 @@
+/*
+ * liblast: GB300 (sm_103a) kernels for LAST's edge-side token selection
+ * ("The Last Query Token Guides Visual Token Pruning ...", Sec. 3.2-3.4).
+ *
+ * The path, per request b of a ragged batch:
+ *   1. last_scores  Eq. 6-8: the attention row of the last query position
+ *                   p* = P_b - 1 (a full softmax over all P_b keys, visual and
+ *                   text, including p* itself) is summed over every layer and
+ *                   q-head at the visual positions and normalised over the
+ *                   visual span: w~_i = s_i / sum_j s_j.
+ *   2. last_select  Eq. 9-11: importance-weighted greedy k-center selection
+ *                   under cosine distance on the encoder features X, budget k_b.
+ *   3. last_gather  Eq. 12: the kept rows of X in ascending index order.
+ *   last_prune runs 1-3 back to back on one stream.
+ *
+ * Conventions shared by every entry point
+ *   - All tensors are DEVICE pointers (caller-allocated, e.g. torch tensors);
+ *     the library allocates no device memory.  Scratch lives in a caller
+ *     workspace of at least last_workspace_size() bytes (256-byte aligned).
+ *   - The offset arrays in last_problem are HOST arrays; each call validates
+ *     them and copies a small plan into the workspace on `stream`.
+ *   - Calls are asynchronous on `stream` (a cudaStream_t; NULL = legacy
+ *     default stream).  Successive calls on one stream may reuse one
+ *     workspace; concurrent calls need distinct workspaces.
+ *   - Argument errors are detected on the host before any launch; the call
+ *     returns a status and touches no output.  Device-side index checks (only
+ *     last_gather takes caller indices) set a flag in the workspace that
+ *     last_poll() reports.
+ *   - The selection is deterministic and, given the same w~, bit-identical to
+ *     the canonical fp32 arithmetic below on every run:
+ *       dot(a,b): lane l in 0..31 owns coordinate groups g = l, l+32, l+64, ...
+ *                 of 8 consecutive coordinates; it accumulates them in
+ *                 increasing coordinate order with one fp32 fma each; the 32
+ *                 lane sums are combined by an xor butterfly (offsets 16..1).
+ *       r_i = dot(x_i,x_i) > 0 ? 1/sqrt(dot(x_i,x_i)) : 0  (IEEE div, sqrt)
+ *       delta_i = min(delta_i, 1 - (dot(x_i,x_j) * r_i) * r_j),  p_i = w~_i * delta_i
+ *       argmax ties go to the lowest index; selected tokens are excluded.
+ *
+ * Layouts (row-major, no padding)
+ *   q      [batch][num_layers][num_q_heads][head_dim]      query of p* per layer
+ *   k      [num_layers][cu_seqlens[batch]][num_kv_heads][head_dim]   packed keys
+ *   x      [cu_vis[batch]][feat_dim]                       encoder features
+ *   w      [cu_vis[batch]] fp32                            w~ (Eq. 8)
+ *   idx    [cu_keep[batch]] int32, request-local, ascending per request
+ *   x_out  [cu_keep[batch]][feat_dim], same dtype as x
+ *   q-head h reads kv-head h / (num_q_heads / num_kv_heads).
+ *
+ * Limits (LAST_ERR_UNSUPPORTED beyond them; last_error_message() says which):
+ *   scoring   G = num_q_heads / num_kv_heads in 1..8; head_dim * elem_bytes is
+ *             16 bytes times a power of two, at most 512 bytes (1024 when G <= 2);
+ *             num_kv_heads * head_dim * elem_bytes small enough that one key's
+ *             row fits one 256-thread CTA pass (e.g. 16 x 128 bf16, 16 x 64 fp32);
+ *             num_layers * num_q_heads <= 6144.
+ *   selection feat_dim a multiple of 8, at most 2048.
+ */
+#ifndef LAST_H_
+#define LAST_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  LAST_OK = 0,
+  LAST_ERR_INVALID_ARG = 1,          /* shape/offset/pointer check failed (host) */
+  LAST_ERR_UNSUPPORTED = 2,          /* valid but outside the compiled limits */
+  LAST_ERR_WORKSPACE_TOO_SMALL = 3,  /* ws_bytes < last_workspace_size() */
+  LAST_ERR_CUDA = 4,                 /* a CUDA runtime call failed */
+  LAST_ERR_DEVICE_INDEX = 5          /* last_poll: a caller index was out of range */
+} last_status;
+
+typedef enum { LAST_DTYPE_F32 = 0, LAST_DTYPE_BF16 = 1 } last_dtype;
+
+/* Problem description (Eq. 2, Eq. 5-7).  Request b has P_b = cu_seqlens[b+1] -
+ * cu_seqlens[b] positions whose last one is the query token p*; its N_b =
+ * cu_vis[b+1] - cu_vis[b] visual tokens occupy positions vis_start[b] ..
+ * vis_start[b] + N_b - 1 (which must end before p*); it keeps
+ * k_b = cu_keep[b+1] - cu_keep[b] tokens, 0 <= k_b <= N_b (Eq. 2; see
+ * last_budget).  All four arrays are host memory, read during the call only. */
+typedef struct {
+  int32_t batch;
+  int32_t num_layers;      /* L: layers whose rows are summed (Eq. 7) */
+  int32_t num_q_heads;     /* H in Eq. 7 */
+  int32_t num_kv_heads;
+  int32_t head_dim;
+  int32_t feat_dim;        /* d_v in Eq. 1 */
+  int32_t dtype;           /* last_dtype of q, k and x */
+  float softmax_scale;     /* <= 0 selects 1/sqrt(head_dim) */
+  const int32_t *cu_seqlens; /* [batch+1], cu_seqlens[0] == 0, non-decreasing */
+  const int32_t *vis_start;  /* [batch] */
+  const int32_t *cu_vis;     /* [batch+1] */
+  const int32_t *cu_keep;    /* [batch+1] */
+} last_problem;
+
+/* Bytes of device workspace every entry point below needs for `p`.
+ * Returns LAST_ERR_INVALID_ARG / LAST_ERR_UNSUPPORTED for a bad problem. */
+last_status last_workspace_size(const last_problem *p, size_t *bytes);
+
+/* Eq. 6-8.  w_out [cu_vis[batch]] fp32 receives w~ (sums to 1 per request). */
+last_status last_scores(const last_problem *p, const void *q, const void *k, float *w_out,
+                        void *ws, size_t ws_bytes, void *stream);
+
+/* Eq. 9-12.  w [cu_vis[batch]] fp32 (e.g. from last_scores); idx_out
+ * [cu_keep[batch]] receives sort(S_K) per request, request-local.  When x_out
+ * is not NULL the kept rows are also written there (the fused form of
+ * last_gather). */
+last_status last_select(const last_problem *p, const float *w, const void *x,
+                        int32_t *idx_out, void *x_out, void *ws, size_t ws_bytes,
+                        void *stream);
+
+/* Eq. 12.  x_out[r] = x[cu_vis[b] + idx[r]] for r in request b's output range.
+ * An index outside [0, N_b) leaves its row unwritten and makes last_poll
+ * return LAST_ERR_DEVICE_INDEX. */
+last_status last_gather(const last_problem *p, const void *x, const int32_t *idx,
+                        void *x_out, void *ws, size_t ws_bytes, void *stream);
+
+/* The whole path: scores, selection, ordered gather.  w_out may be NULL (w~
+ * is then kept in the workspace); x_out may be NULL (indices only). */
+last_status last_prune(const last_problem *p, const void *q, const void *k, const void *x,
+                       float *w_out, int32_t *idx_out, void *x_out,
+                       void *ws, size_t ws_bytes, void *stream);
+
+/* Synchronises `stream`, then reports the device-side flag of the last call
+ * that used `ws` (LAST_OK or LAST_ERR_DEVICE_INDEX). */
+last_status last_poll(const void *ws, void *stream);
+
+/* Eq. 2: k = ceil(num * n_vis / den) in exact integer arithmetic
+ * (rho = num/den); -1 for n_vis < 0, num < 0 or den <= 0. */
+int32_t last_budget(int32_t n_vis, int32_t num, int32_t den);
+
+const char *last_status_string(last_status s);
+
+/* Human-readable detail of the last non-OK status returned on this thread. */
+const char *last_error_message(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* LAST_H_ */

@@ -1,0 +1,72 @@
+// Host-side plan shared by the entry points and the kernel launchers.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cstddef>
+#include <cstdint>
+#include <string>
+#include <vector>
+
+#include "last.h"
+
+namespace last {
+
+// Per-request metadata row staged into the workspace (int32 each).
+enum MetaField : int {
+  kSeqStart = 0,   // cu_seqlens[b]
+  kSeqLen,         // P_b
+  kVisStart,       // v_b (position of the first visual token)
+  kVisOff,         // cu_vis[b]
+  kNumVis,         // N_b
+  kKeepOff,        // cu_keep[b]
+  kNumKeep,        // k_b
+  kChunkBase,      // first score chunk of request b
+  kMetaFields
+};
+
+constexpr int kScoreChunk = 128;     // keys per scoring CTA
+constexpr int kScoreThreads = 256;
+constexpr int kReduceThreads = 512;
+constexpr int kMaxGroup = 8;         // q-heads per kv-head supported by the scoring kernel
+constexpr int kMaxFeatDim = 2048;    // selection keeps x_j in 64 fp32 registers per lane
+constexpr int kSelectWarps = 8;
+constexpr int kGatherThreads = 256;
+
+// Device error flags (first word of the workspace).
+constexpr unsigned kErrGatherIndex = 1u;
+
+struct Plan {
+  // problem
+  int B = 0, L = 0, Hq = 0, Hkv = 0, D = 0, dv = 0, dtype = 0;
+  int G = 0, elem = 0;
+  float scale = 0.f;
+  long long total_keys = 0, total_vis = 0, total_keep = 0;
+  int max_seq = 0, max_vis = 0, max_keep = 0;
+  int total_chunks = 0;
+  // workspace byte offsets
+  size_t off_err = 0, off_meta = 0, off_items = 0, off_order = 0;
+  size_t off_stats = 0, off_zlog = 0, off_w = 0, total_bytes = 0;
+  // host staging (meta rows, score items, selection order) in ws order
+  std::vector<int32_t> host_blob;
+  size_t blob_bytes = 0;  // bytes from off_meta to the end of the order array
+};
+
+// Validation + layout.  `need_scores` / `need_select` widen the checks to the
+// parts a call uses.  Returns LAST_OK or an error with a message set.
+last_status make_plan(const last_problem *p, bool need_scores, bool need_select, Plan *plan);
+
+void set_error(const std::string &msg);
+
+// Kernel launchers (return cudaSuccess or the launch error).
+cudaError_t launch_scores(const Plan &pl, const void *q, const void *k, float *w_out,
+                          char *ws, cudaStream_t s);
+cudaError_t launch_select(const Plan &pl, const float *w, const void *x, int32_t *idx_out,
+                          void *x_out, char *ws, cudaStream_t s);
+cudaError_t launch_gather(const Plan &pl, const void *x, const int32_t *idx, void *x_out,
+                          char *ws, cudaStream_t s);
+
+// Checks the compiled limits of the scoring / selection kernels.
+bool scores_supported(const Plan &pl, std::string *why);
+bool select_supported(const Plan &pl, std::string *why);
+
+}  // namespace last

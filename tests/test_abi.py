@@ -1,0 +1,115 @@
+"""CPU-side checks of the C ABI: the library loads, exports every function the
+public header declares, and rejects bad problems on the host before touching
+the GPU (no compute call runs here)."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+import paper_2607_27952_gb300 as last
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "last.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2607_27952_gb300.build import build
+    build()
+    return last.load_library()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(last_[a-z_]+)\s*\(", text)))
+
+
+def test_every_declared_symbol_is_exported(lib):
+    names = declared_functions()
+    assert len(names) >= 9
+    for n in names:
+        assert hasattr(lib, n), f"{n} declared in include/last.h but not exported"
+    assert set(names) == set(last.EXPORTED)
+
+
+def _problem(**kw):
+    base = dict(batch=2, num_layers=1, num_q_heads=4, num_kv_heads=2, head_dim=64, feat_dim=256,
+                dtype="bf16", cu_seqlens=[0, 10, 30], vis_start=[0, 2], cu_vis=[0, 6, 14],
+                cu_keep=[0, 2, 5])
+    base.update(kw)
+    return last.Problem(**base)
+
+
+def test_workspace_size_is_host_only(lib):
+    n = last.last_workspace_size(_problem())
+    assert n > 0 and n % 256 == 0
+    bigger = last.last_workspace_size(_problem(cu_seqlens=[0, 3000, 7000]))
+    assert bigger > n
+
+
+@pytest.mark.parametrize("kw,status", [
+    (dict(num_q_heads=6, num_kv_heads=4), last.LAST_ERR_INVALID_ARG),       # Hq % Hkv
+    (dict(vis_start=[4, 2]), last.LAST_ERR_INVALID_ARG),                     # span reaches p*
+    (dict(cu_keep=[0, 7, 9]), last.LAST_ERR_INVALID_ARG),                    # k_b > N_b
+    (dict(cu_keep=[0, 3, 2]), last.LAST_ERR_INVALID_ARG),                    # k_b < 0
+    (dict(cu_seqlens=[0, 0, 30], vis_start=[0, 2], cu_vis=[0, 0, 14],
+          cu_keep=[0, 0, 5]), last.LAST_ERR_INVALID_ARG),                    # P_b = 0
+    (dict(num_q_heads=18, num_kv_heads=2), last.LAST_ERR_UNSUPPORTED),       # G = 9 > 8
+    (dict(head_dim=80), last.LAST_ERR_UNSUPPORTED),                          # 160 B rows
+])
+def test_scores_rejects_bad_problems_before_launch(lib, kw, status):
+    prob = _problem(**kw)
+    with pytest.raises(last.LastError) as e:
+        last.last_scores(prob, 16, 16, 16, (256, 1 << 30), stream=0)
+    assert e.value.status == status
+
+
+@pytest.mark.parametrize("kw,status", [
+    (dict(feat_dim=100), last.LAST_ERR_INVALID_ARG),
+    (dict(feat_dim=4096), last.LAST_ERR_UNSUPPORTED),
+    (dict(cu_vis=[0, 6, 5]), last.LAST_ERR_INVALID_ARG),
+])
+def test_select_rejects_bad_problems_before_launch(lib, kw, status):
+    prob = _problem(**kw)
+    with pytest.raises(last.LastError) as e:
+        last.last_select(prob, 16, 16, 16, (256, 1 << 30), stream=0, x_out=None)
+    assert e.value.status == status
+
+
+def test_workspace_checks(lib):
+    prob = _problem()
+    need = last.last_workspace_size(prob)
+    with pytest.raises(last.LastError) as e:
+        last.last_prune(prob, 16, 16, 16, None, 16, None, (256, need - 1), stream=0)
+    assert e.value.status == last.LAST_ERR_WORKSPACE_TOO_SMALL
+    with pytest.raises(last.LastError) as e:
+        last.last_prune(prob, 16, 16, 16, None, 16, None, (8, need), stream=0)
+    assert e.value.status == last.LAST_ERR_INVALID_ARG      # not 256-byte aligned
+    with pytest.raises(last.LastError) as e:
+        last.last_prune(prob, 16, 24, 16, None, 16, None, (256, need), stream=0)
+    assert e.value.status == last.LAST_ERR_INVALID_ARG      # k not 16-byte aligned
+
+
+@pytest.mark.parametrize("n,num,den", [(576, 1, 8), (16384, 1, 20), (16384, 1, 4), (257, 1, 8),
+                                       (0, 1, 8), (2880, 1, 8), (4095, 1, 8), (7, 3, 3)])
+def test_budget_matches_ceil(lib, n, num, den):
+    import math
+    from fractions import Fraction
+    assert last.last_budget(n, num, den) == math.ceil(Fraction(num * n, den))
+
+
+def test_budget_rejects_bad_ratio(lib):
+    assert last.last_budget(-1, 1, 8) == -1
+    assert last.last_budget(10, 1, 0) == -1
+
+
+def test_status_strings(lib):
+    for st in range(6):
+        assert last.last_status_string(st).startswith("LAST_")
+
+
+def test_library_path_is_in_tree(lib):
+    assert os.path.dirname(last.LIB_PATH) == os.path.join(ROOT, "paper_2607_27952_gb300")

@@ -1,0 +1,236 @@
+"""GPU parity against the oracle through the C ABI (Eq. 6-12).
+
+Rules: scores within rtol 1e-3 of the fp64 oracle; kept indices and gathered
+rows bit-exact against the canonical-fp32 oracle selection when run on the same
+scores (ties -> lowest index); end-to-end, an index sequence may leave the
+oracle's only at a near-tie (products within 1e-3).
+"""
+import numpy as np
+import pytest
+
+import oracle
+from workloads import config, custom
+
+from gpu_util import (DeviceWorkload, assert_gather_equal, assert_scores_close,
+                      assert_selection_equal, assert_valid_selection, near_tie_divergence,
+                      oracle_selection)
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("needs a GPU")
+    from paper_2607_27952_gb300.build import build
+    import paper_2607_27952_gb300 as last
+    build()
+    last.load_library()
+    oracle.build()
+
+
+# Oracle-sized cases: several tiles (16-CTA clusters, 128-key chunks), ragged tails.
+MINI = {
+    "c1": lambda: config("c1"),
+    "c2": lambda: config("c2", batch=6, budget="mixed"),
+    "c3": lambda: config("c3", batch=2, n_vis=1152),
+    "c4": lambda: config("c4", batch=8, n_vis=[300, 1024, 257, 777, 513, 260, 999, 640]),
+    "c5": lambda: config("c5", batch=2, n_vis=2048, budget=12.5),
+    "gqa7_d64": lambda: custom(name="qwen2-0.5b-like", seed=31, batch=3, n_vis=[256, 143, 401],
+                               n_text=[20, 7, 33], n_before=[14, 3, 0], num_layers=3,
+                               num_q_heads=14, num_kv_heads=2, head_dim=64, feat_dim=1024,
+                               dtype="bf16", keep=[32, 18, 50], n_clusters=16, n_planted=5),
+    "f32_ragged_d1000": lambda: custom(name="f32-d1000", seed=32, batch=4, n_vis=[65, 1, 300, 17],
+                                       n_text=[1, 3, 2, 5], n_before=[0, 2, 7, 1], num_layers=2,
+                                       num_q_heads=8, num_kv_heads=8, head_dim=32,
+                                       feat_dim=1000, dtype="f32", keep=[9, 1, 38, 17],
+                                       n_clusters=6, n_planted=3),
+}
+
+
+@pytest.mark.parametrize("name", list(MINI))
+def test_scores_match_oracle(name):
+    wl = MINI[name]()
+    w_ref = oracle.scores(wl.q, wl.k, wl.cu_seqlens, wl.vis_start, wl.cu_vis,
+                          num_kv_heads=wl.num_kv_heads, scale=wl.scale)
+    w_gpu = DeviceWorkload(wl).scores()
+    assert_scores_close(w_gpu, w_ref, wl)
+
+
+@pytest.mark.parametrize("name", list(MINI))
+def test_select_bitexact_on_oracle_scores(name):
+    wl = MINI[name]()
+    w32 = oracle.scores(wl.q, wl.k, wl.cu_seqlens, wl.vis_start, wl.cu_vis,
+                        num_kv_heads=wl.num_kv_heads, scale=wl.scale).astype(np.float32)
+    idx = DeviceWorkload(wl).select(w32)
+    assert_valid_selection(wl, idx)
+    assert_selection_equal(wl, w32, idx, range(wl.batch))
+
+
+@pytest.mark.parametrize("name", list(MINI))
+def test_prune_end_to_end(name):
+    wl = MINI[name]()
+    dw = DeviceWorkload(wl)
+    w_gpu, idx, xs = dw.prune()
+    w64 = oracle.scores(wl.q, wl.k, wl.cu_seqlens, wl.vis_start, wl.cu_vis,
+                        num_kv_heads=wl.num_kv_heads, scale=wl.scale)
+    assert_scores_close(w_gpu, w64, wl)
+    assert_valid_selection(wl, idx)
+    # bit-exact on the GPU's own scores, and the rows are a bitwise gather
+    assert_selection_equal(wl, w_gpu, idx, range(wl.batch))
+    assert_gather_equal(wl, idx, xs, range(wl.batch))
+    # against the oracle's scores: sequences may part only at a near-tie
+    w32 = w64.astype(np.float32)
+    for b in range(wl.batch):
+        v0, v1 = wl.cu_vis[b], wl.cu_vis[b + 1]
+        ref = oracle_selection(wl, w32, b)
+        alt = oracle_selection(wl, w_gpu, b)
+        d = near_tie_divergence(wl.x[v0:v1], w64[v0:v1], ref, alt)
+        assert d is None or d[1] <= 1e-3, f"request {b}: diverged at step {d[0]} with gap {d[1]}"
+
+
+def test_prune_is_deterministic():
+    wl = MINI["c4"]()
+    dw = DeviceWorkload(wl)
+    a = dw.prune()
+    for _ in range(3):
+        b = dw.prune()
+        for u, v in zip(a, b):
+            assert np.array_equal(u.view(np.uint8), v.view(np.uint8))
+
+
+def test_budget_edge_cases():
+    """k = 0, k = N, N = 0, N smaller than the cluster, N = 1, in one ragged batch."""
+    wl = custom(name="edges", seed=41, batch=7, n_vis=[0, 5, 40, 1, 300, 16, 33],
+                n_text=[1, 2, 1, 3, 4, 1, 2], n_before=[0, 1, 0, 0, 9, 0, 2], num_layers=1,
+                num_q_heads=4, num_kv_heads=4, head_dim=64, feat_dim=256, dtype="bf16",
+                keep=[0, 5, 0, 1, 299, 3, 33], n_clusters=4, n_planted=2)
+    dw = DeviceWorkload(wl)
+    w_gpu, idx, xs = dw.prune()
+    assert_valid_selection(wl, idx)
+    assert_selection_equal(wl, w_gpu, idx, range(wl.batch))
+    assert_gather_equal(wl, idx, xs, range(wl.batch))
+    k0, k1 = wl.cu_keep[1], wl.cu_keep[2]
+    assert idx[k0:k1].tolist() == list(range(5))           # k = N keeps everything
+    k0, k1 = wl.cu_keep[6], wl.cu_keep[7]
+    assert idx[k0:k1].tolist() == list(range(33))
+
+
+@pytest.mark.parametrize("dv", [8, 264, 1536, 2048])
+def test_feature_widths(dv):
+    wl = custom(name=f"dv{dv}", seed=50 + dv, batch=3, n_vis=[130, 77, 250], n_text=[3, 3, 3],
+                num_layers=1, num_q_heads=2, num_kv_heads=1, head_dim=64, feat_dim=dv,
+                dtype="bf16", keep=[20, 9, 61], n_clusters=8, n_planted=2)
+    dw = DeviceWorkload(wl)
+    w_gpu, idx, xs = dw.prune()
+    assert_selection_equal(wl, w_gpu, idx, range(wl.batch))
+    assert_gather_equal(wl, idx, xs, range(wl.batch))
+
+
+def test_identical_and_orthogonal_features():
+    """Special cases with textbook answers run through the kernels."""
+    import torch
+    N, d = 300, 1024
+    x = np.zeros((N, d), np.float32)
+    x[:, :] = 1.0                                          # identical rows, cos = 1 exactly
+    wl = custom(name="ident", seed=60, batch=1, n_vis=N, n_text=2, num_layers=1, num_q_heads=2,
+                num_kv_heads=2, head_dim=64, feat_dim=d, dtype="f32", keep=[12])
+    wl.x = x
+    w = np.random.default_rng(0).dirichlet(np.ones(N)).astype(np.float32)
+    idx = DeviceWorkload(wl).select(w)
+    j1 = int(np.argmax(w))
+    want = sorted([j1] + [i for i in range(N) if i != j1][:11])
+    assert idx.tolist() == want
+    # orthogonal rows: the greedy is top-k of w
+    x2 = np.zeros((N, d), np.float32)
+    x2[np.arange(N), np.random.default_rng(1).permutation(d)[:N]] = 2.0
+    wl.x = x2
+    idx2 = DeviceWorkload(wl).select(w)
+    assert idx2.tolist() == sorted(np.argsort(-w, kind="stable")[:12].tolist())
+
+
+def test_gather_and_device_index_flag():
+    import torch
+    import paper_2607_27952_gb300 as last
+    from gpu_util import problem_of, to_dev, to_host_bits
+    wl = custom(name="gather", seed=70, batch=3, n_vis=[50, 9, 120], n_text=[1, 1, 1],
+                feat_dim=1536, dtype="bf16", keep=[7, 0, 30])
+    prob = problem_of(wl)
+    dev = torch.device("cuda:0")
+    rng = np.random.default_rng(0)
+    idx = np.concatenate([np.sort(rng.choice(50, 7, replace=False)),
+                          rng.choice(120, 30, replace=True)]).astype(np.int32)
+    x = to_dev(wl.x, dev)
+    out = torch.zeros((37, 1536), dtype=torch.bfloat16, device=dev)
+    ws = last.workspace(prob, dev)
+    last.last_gather(prob, x, torch.from_numpy(idx).to(dev), out, ws)
+    last.last_poll(ws)
+    got = to_host_bits(out)
+    assert np.array_equal(got[:7], wl.x[:50][idx[:7]])
+    assert np.array_equal(got[7:], wl.x[59:179][idx[7:]])
+    bad = idx.copy()
+    bad[3] = 50                                            # out of range for request 0
+    out.zero_()
+    last.last_gather(prob, x, torch.from_numpy(bad).to(dev), out, ws)
+    with pytest.raises(last.LastError) as e:
+        last.last_poll(ws)
+    assert e.value.status == last.LAST_ERR_DEVICE_INDEX
+    got = to_host_bits(out)
+    assert not got[3].any() and np.array_equal(got[4:7], wl.x[:50][bad[4:7]])
+    last.last_gather(prob, x, torch.from_numpy(idx).to(dev), out, ws)
+    last.last_poll(ws)                                     # flag cleared by the next call
+
+
+# ---- full sizes: scores everywhere, selection on sampled requests ----
+FULL = {
+    "c1": (lambda: config("c1"), None),
+    "c2_k64": (lambda: config("c2", budget=64), [0, 31, 63]),
+    "c2_k128": (lambda: config("c2", budget=128), [0, 17, 40]),
+    "c2_k192": (lambda: config("c2", budget=192), [5, 63]),
+    "c3": (lambda: config("c3"), [0]),
+    "c4": (lambda: config("c4"), "longest+2"),
+}
+
+
+@pytest.mark.parametrize("name", list(FULL))
+def test_full_size(name):
+    make, sample = FULL[name]
+    wl = make()
+    dw = DeviceWorkload(wl)
+    w_gpu, idx, xs = dw.prune()
+    w64 = oracle.scores(wl.q, wl.k, wl.cu_seqlens, wl.vis_start, wl.cu_vis,
+                        num_kv_heads=wl.num_kv_heads, scale=wl.scale)
+    assert_scores_close(w_gpu, w64, wl)
+    assert_valid_selection(wl, idx)
+    if sample is None:
+        reqs = range(wl.batch)
+    elif sample == "longest+2":
+        n = np.diff(wl.cu_vis)
+        reqs = [int(np.argmax(n)), int(np.argmin(n)), wl.batch // 2]
+    else:
+        reqs = sample
+    assert_selection_equal(wl, w_gpu, idx, reqs)
+    assert_gather_equal(wl, idx, xs, range(wl.batch))
+
+
+@pytest.mark.parametrize("pct", [5, 12.5, 25])
+def test_full_size_video(pct):
+    """c5 at full size.  The greedy sequence does not depend on k (Eq. 9-11), so the
+    kept set for a small budget k' is a prefix of the one for k: the oracle checks the
+    k' = 40 selection of two requests exactly, and the full-budget result must contain it."""
+    wl = config("c5", budget=pct)
+    dw = DeviceWorkload(wl)
+    w_gpu, idx, xs = dw.prune()
+    w64 = oracle.scores(wl.q, wl.k, wl.cu_seqlens, wl.vis_start, wl.cu_vis,
+                        num_kv_heads=wl.num_kv_heads, scale=wl.scale)
+    assert_scores_close(w_gpu, w64, wl)
+    assert_valid_selection(wl, idx)
+    assert_gather_equal(wl, idx, xs, range(wl.batch))
+    kp = 40
+    small = np.arange(wl.batch + 1, dtype=np.int32) * kp
+    idx_small = dw.select(w_gpu, cu_keep=small)
+    assert_selection_equal(wl, w_gpu, idx_small, [0, 5], cu_keep=small)
+    for b in range(wl.batch):
+        big = idx[wl.cu_keep[b]:wl.cu_keep[b + 1]]
+        assert np.isin(idx_small[small[b]:small[b + 1]], big).all(), f"request {b}: not a prefix"
