@@ -23,9 +23,10 @@
  *     default stream).  Successive calls on one stream may reuse one
  *     workspace; concurrent calls need distinct workspaces.
  *   - Argument errors are detected on the host before any launch; the call
- *     returns a status and touches no output.  Device-side index checks (only
- *     last_gather takes caller indices) set a flag in the workspace that
- *     last_poll() reports.
+ *     returns a status and touches no output.  Device-side checks set a flag in
+ *     the workspace that last_poll() reports: an out-of-range caller index
+ *     (last_gather) or an expired bounded wait (every device wait has an
+ *     iteration limit, so no call can hang the GPU).
  *   - The selection is deterministic and, given the same w~, bit-identical to
  *     the canonical fp32 arithmetic below on every run:
  *       dot(a,b): lane l in 0..31 owns coordinate groups g = l, l+32, l+64, ...
@@ -69,7 +70,8 @@ typedef enum {
   LAST_ERR_UNSUPPORTED = 2,          /* valid but outside the compiled limits */
   LAST_ERR_WORKSPACE_TOO_SMALL = 3,  /* ws_bytes < last_workspace_size() */
   LAST_ERR_CUDA = 4,                 /* a CUDA runtime call failed */
-  LAST_ERR_DEVICE_INDEX = 5          /* last_poll: a caller index was out of range */
+  LAST_ERR_DEVICE_INDEX = 5,         /* last_poll: a caller index was out of range */
+  LAST_ERR_TIMEOUT = 6               /* last_poll: a bounded device wait expired; outputs invalid */
 } last_status;
 
 typedef enum { LAST_DTYPE_F32 = 0, LAST_DTYPE_BF16 = 1 } last_dtype;
@@ -123,8 +125,10 @@ last_status last_prune(const last_problem *p, const void *q, const void *k, cons
                        float *w_out, int32_t *idx_out, void *x_out,
                        void *ws, size_t ws_bytes, void *stream);
 
-/* Synchronises `stream`, then reports the device-side flag of the last call
- * that used `ws` (LAST_OK or LAST_ERR_DEVICE_INDEX). */
+/* Synchronises `stream`, then reports the device-side flags of the last call
+ * that used `ws`: LAST_OK, LAST_ERR_DEVICE_INDEX, or LAST_ERR_TIMEOUT (a wait
+ * on an asynchronous copy gave up after its iteration limit instead of hanging;
+ * the outputs of that call are then invalid). */
 last_status last_poll(const void *ws, void *stream);
 
 /* Eq. 2: k = ceil(num * n_vis / den) in exact integer arithmetic

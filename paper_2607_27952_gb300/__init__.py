@@ -26,6 +26,7 @@ LAST_ERR_UNSUPPORTED = 2
 LAST_ERR_WORKSPACE_TOO_SMALL = 3
 LAST_ERR_CUDA = 4
 LAST_ERR_DEVICE_INDEX = 5
+LAST_ERR_TIMEOUT = 6
 
 LAST_DTYPE_F32 = 0
 LAST_DTYPE_BF16 = 1

@@ -282,6 +282,8 @@ last_status last_poll(const void *ws, void *stream) {
   cudaError_t e = cudaMemcpyAsync(&flag, ws, sizeof flag, cudaMemcpyDeviceToHost, s);
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
   if (e != cudaSuccess) return cuda_fail(e, "poll");
+  if (flag & kErrTimeout)
+    return fail(LAST_ERR_TIMEOUT, "a bounded device wait expired; outputs of that call are invalid");
   if (flag & kErrGatherIndex)
     return fail(LAST_ERR_DEVICE_INDEX, "a gather index was outside [0, N_b)");
   return LAST_OK;
@@ -303,6 +305,7 @@ const char *last_status_string(last_status s) {
     case LAST_ERR_WORKSPACE_TOO_SMALL: return "LAST_ERR_WORKSPACE_TOO_SMALL";
     case LAST_ERR_CUDA: return "LAST_ERR_CUDA";
     case LAST_ERR_DEVICE_INDEX: return "LAST_ERR_DEVICE_INDEX";
+    case LAST_ERR_TIMEOUT: return "LAST_ERR_TIMEOUT";
   }
   return "LAST_ERR_UNKNOWN";
 }

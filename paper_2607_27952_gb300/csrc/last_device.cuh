@@ -41,6 +41,16 @@ __device__ __forceinline__ U4 ldg(const void *p) {
 __device__ __forceinline__ U4 lds(const void *p) {
   return *reinterpret_cast<const U4 *>(p);
 }
+// 16-byte shared-memory load from a 32-bit shared-window address.
+__device__ __forceinline__ U4 lds32(uint32_t addr) {
+  U4 r;
+  asm volatile("ld.shared.v4.u32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w) : "r"(addr));
+  return r;
+}
+__device__ __forceinline__ uint32_t smem_addr(const void *p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
 
 // ---- argmax keys: (ordered fp32 bits << 32) | (0xffffffff - index) ----
 // Larger key = larger value; equal values prefer the lower index.  -0 is
@@ -56,6 +66,11 @@ __device__ __forceinline__ int key_index(unsigned long long key) {
   return static_cast<int>(0xffffffffu - static_cast<uint32_t>(key & 0xffffffffull));
 }
 
+__device__ __forceinline__ unsigned long long shfl_u64(unsigned long long v, int src) {
+  uint32_t lo = __shfl_sync(0xffffffffu, static_cast<uint32_t>(v), src);
+  uint32_t hi = __shfl_sync(0xffffffffu, static_cast<uint32_t>(v >> 32), src);
+  return (static_cast<unsigned long long>(hi) << 32) | lo;
+}
 __device__ __forceinline__ unsigned long long shfl_xor_u64(unsigned long long v, int o) {
   uint32_t lo = __shfl_xor_sync(0xffffffffu, static_cast<uint32_t>(v), o);
   uint32_t hi = __shfl_xor_sync(0xffffffffu, static_cast<uint32_t>(v >> 32), o);
@@ -89,6 +104,10 @@ __device__ __forceinline__ void st_cluster_u64(uint32_t addr, unsigned long long
 __device__ __forceinline__ void st_cluster_f32(uint32_t addr, float v) {
   asm volatile("st.shared::cluster.f32 [%0], %1;" :: "r"(addr), "f"(v) : "memory");
 }
+__device__ __forceinline__ void st_cluster_v4f(uint32_t addr, float4 v) {
+  asm volatile("st.shared::cluster.v4.f32 [%0], {%1,%2,%3,%4};"
+               :: "r"(addr), "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w) : "memory");
+}
 __device__ __forceinline__ void st_cluster_s32(uint32_t addr, int v) {
   asm volatile("st.shared::cluster.s32 [%0], %1;" :: "r"(addr), "r"(v) : "memory");
 }
@@ -97,6 +116,43 @@ __device__ __forceinline__ U4 ld_cluster_v4(uint32_t addr) {
   asm volatile("ld.shared::cluster.v4.u32 {%0,%1,%2,%3}, [%4];"
                : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w) : "r"(addr) : "memory");
   return r;
+}
+
+// ---- mbarrier + TMA bulk copies (global -> this CTA's shared memory) ----
+__device__ __forceinline__ void mbar_init(unsigned long long *bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" :: "r"(smem_addr(bar)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void fence_mbar_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(unsigned long long *bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;"
+               :: "r"(smem_addr(bar)), "r"(bytes) : "memory");
+}
+// 1-D bulk copy; dst, src and bytes must be multiples of 16.
+__device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t bytes,
+                                         unsigned long long *bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+               :: "r"(smem_addr(dst)), "l"(src), "r"(bytes), "r"(smem_addr(bar)) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(unsigned long long *bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile("{\n\t.reg .pred p;\n\t"
+               "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+               "selp.u32 %0, 1, 0, p;\n\t}"
+               : "=r"(ok) : "r"(smem_addr(bar)), "r"(parity) : "memory");
+  return ok != 0;
+}
+// Waits for phase `parity` of `bar` with an iteration limit; on expiry sets
+// `flag` in *err and returns false (the caller carries on with whatever data
+// arrived, so the kernel always terminates).
+constexpr uint32_t kWaitLimit = 1u << 22;
+__device__ __forceinline__ bool mbar_wait_bounded(unsigned long long *bar, uint32_t parity,
+                                                  unsigned *err, unsigned flag) {
+  for (uint32_t i = 0; i < kWaitLimit; ++i)
+    if (mbar_try_wait(bar, parity)) return true;
+  atomicOr(err, flag);
+  return false;
 }
 
 }  // namespace last

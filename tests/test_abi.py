@@ -107,7 +107,7 @@ def test_budget_rejects_bad_ratio(lib):
 
 
 def test_status_strings(lib):
-    for st in range(6):
+    for st in range(7):
         assert last.last_status_string(st).startswith("LAST_")
 
 
