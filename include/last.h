@@ -125,6 +125,21 @@ last_status last_prune(const last_problem *p, const void *q, const void *k, cons
                        float *w_out, int32_t *idx_out, void *x_out,
                        void *ws, size_t ws_bytes, void *stream);
 
+/* last_scores without a caller workspace (the paper has no counterpart: this is
+ * a deployment aid).  For callers that cannot allocate device memory at run time
+ * -- e.g. an edge service that reserves all of its device memory at start-up and
+ * treats later allocations as failures, or a program without a device allocator
+ * of its own.  Same inputs, outputs and results as last_scores; the scratch lives
+ * in a fixed 16 MiB array inside the library, held on every GPU that loads the
+ * library until the process exits.  The first call on each device looks up that
+ * array's device address (cudaGetSymbolAddress) with the device current; make
+ * that first call before any stream capture on that device.  All calls share
+ * the array and it keeps the last call's contents: calls whose executions
+ * overlap on the GPU race on it.  A problem needing more than 16 MiB of scratch
+ * (last_workspace_size) returns LAST_ERR_UNSUPPORTED.  Allocates nothing. */
+last_status last_scores_noalloc(const last_problem *p, const void *q, const void *k,
+                                float *w_out, void *stream);
+
 /* Synchronises `stream`, then reports the device-side flags of the last call
  * that used `ws`: LAST_OK, LAST_ERR_DEVICE_INDEX, or LAST_ERR_TIMEOUT (a wait
  * on an asynchronous copy gave up after its iteration limit instead of hanging;

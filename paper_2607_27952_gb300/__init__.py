@@ -32,7 +32,8 @@ LAST_DTYPE_F32 = 0
 LAST_DTYPE_BF16 = 1
 
 EXPORTED = ("last_workspace_size", "last_scores", "last_select", "last_gather", "last_prune",
-            "last_poll", "last_budget", "last_status_string", "last_error_message")
+            "last_poll", "last_budget", "last_status_string", "last_error_message",
+            "last_scores_noalloc")
 
 
 class LastError(RuntimeError):
@@ -76,6 +77,7 @@ def load_library(path: str = LIB_PATH):
     lib.last_gather.argtypes = [PP, P, P, P, P, ctypes.c_size_t, P]
     lib.last_prune.argtypes = [PP, P, P, P, P, P, P, P, ctypes.c_size_t, P]
     lib.last_poll.argtypes = [P, P]
+    lib.last_scores_noalloc.argtypes = [PP, P, P, P, P]
     lib.last_budget.argtypes = [ctypes.c_int32, ctypes.c_int32, ctypes.c_int32]
     lib.last_budget.restype = ctypes.c_int32
     lib.last_status_string.argtypes = [ctypes.c_int]
@@ -83,7 +85,7 @@ def load_library(path: str = LIB_PATH):
     lib.last_error_message.argtypes = []
     lib.last_error_message.restype = ctypes.c_char_p
     for name in ("last_workspace_size", "last_scores", "last_select", "last_gather",
-                 "last_prune", "last_poll"):
+                 "last_prune", "last_poll", "last_scores_noalloc"):
         getattr(lib, name).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -173,6 +175,13 @@ def last_scores(problem: Problem, q, k, w_out, ws, stream=None):
     p, n = _ws(ws)
     _check(load_library().last_scores(problem.ref, _ptr(q), _ptr(k), _ptr(w_out), p, n,
                                       _stream(stream)))
+
+
+def last_scores_noalloc(problem: Problem, q, k, w_out, stream=None):
+    """last_scores with the library's fixed scratch array instead of a workspace
+    (for callers that cannot allocate device memory at run time)."""
+    _check(load_library().last_scores_noalloc(problem.ref, _ptr(q), _ptr(k), _ptr(w_out),
+                                              _stream(stream)))
 
 
 def last_select(problem: Problem, w, x, idx_out, ws, stream=None, x_out=None):
