@@ -28,6 +28,26 @@ template <> struct Elem<__nv_bfloat16> {
   }
 };
 
+// c + a * b with a, b the bf16 in the low/high halves of 32-bit words and fp32
+// c, d: the product is exact in fp32 and the sum is rounded once, so this equals
+// fmaf(widen(a), widen(b), c) bit for bit, without the widening instructions.
+__device__ __forceinline__ float fma_bf16_lo(uint32_t a, uint32_t b, float c) {
+  float d;
+  asm("{\n\t.reg .b16 al, ah, bl, bh;\n\t"
+      "mov.b32 {al, ah}, %1;\n\tmov.b32 {bl, bh}, %2;\n\t"
+      "fma.rn.f32.bf16 %0, al, bl, %3;\n\t}"
+      : "=f"(d) : "r"(a), "r"(b), "f"(c));
+  return d;
+}
+__device__ __forceinline__ float fma_bf16_hi(uint32_t a, uint32_t b, float c) {
+  float d;
+  asm("{\n\t.reg .b16 al, ah, bl, bh;\n\t"
+      "mov.b32 {al, ah}, %1;\n\tmov.b32 {bl, bh}, %2;\n\t"
+      "fma.rn.f32.bf16 %0, ah, bh, %3;\n\t}"
+      : "=f"(d) : "r"(a), "r"(b), "f"(c));
+  return d;
+}
+
 // Read-only streaming load that does not allocate in L1.
 __device__ __forceinline__ U4 ldg_stream(const void *p) {
   U4 r;
@@ -116,6 +136,18 @@ __device__ __forceinline__ U4 ld_cluster_v4(uint32_t addr) {
   asm volatile("ld.shared::cluster.v4.u32 {%0,%1,%2,%3}, [%4];"
                : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w) : "r"(addr) : "memory");
   return r;
+}
+
+// ---- per-thread async copies (global -> shared), grouped ----
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void *src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" :: "r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" :: "n"(N) : "memory");
 }
 
 // ---- mbarrier + TMA bulk copies (global -> this CTA's shared memory) ----

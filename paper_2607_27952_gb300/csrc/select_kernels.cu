@@ -47,6 +47,7 @@ constexpr int kMaxCluster = 16;
 constexpr int kLcap = 16;                          // candidate list length
 constexpr int kTopM = 9;                           // per-warp / per-CTA ranked keys (<= 8 + bound)
 constexpr int kMaxPairs = kLcap * (kLcap - 1) / 2;
+constexpr int kRing = 4;                           // async-copy ring depth (groups in flight)
 
 struct SelectArgs {
   const void *x;
@@ -57,20 +58,32 @@ struct SelectArgs {
   const int32_t *order;  // cluster -> request (most work first)
   int dv, row_bytes, tpc_max, cache_rows, csize;
   int mc;                // candidates each CTA publishes per round (<= kTopM - 1)
+  int ring;              // 1: rows beyond the resident cache stream through an async-copy ring
   unsigned *err;         // workspace error word
 };
 
 // Shared-memory carve-up, identical on host (sizing) and device.
 struct SelectSmem {
-  size_t xcache, cbuf, w, r, dl, list, sel, wtop, pub_key, pub_f, lp_key, lp_f, lp_idx, lp_row,
-      pair, acc, misc, bar, cnt, total;
+  size_t xcache, cbuf, ring, blk, w, r, dl, list, sel, wtop, pub_key, pub_f, lp_key, lp_f, lp_idx,
+      lp_row, pair, acc, misc, bar, cnt, total;
 };
 __host__ __device__ inline size_t align16(size_t v) { return (v + 15) & ~size_t(15); }
-__host__ __device__ inline SelectSmem select_smem(int cache_rows, int row_bytes, int tpc_max) {
+// Bytes of the per-warp async-copy rings: kRing groups x tb rows x (8 coordinates x
+// elem bytes) per lane.
+__host__ __device__ inline size_t ring_bytes(int ring, int tb, int elem) {
+  return ring ? (size_t)kSelectWarps * kRing * tb * 8 * elem * 32 : 0;
+}
+__host__ __device__ inline int blocks_per_warp(int tpc_max, int tb) {
+  return (tpc_max + kSelectWarps * tb - 1) / (kSelectWarps * tb);
+}
+__host__ __device__ inline SelectSmem select_smem(int cache_rows, int row_bytes, int tpc_max,
+                                                  int ring, int tb, int elem) {
   SelectSmem s;
   size_t o = 0;
   s.xcache = o; o += (size_t)cache_rows * row_bytes;
   s.cbuf = o; o += (size_t)kLcap * row_bytes;
+  s.ring = o; o += ring_bytes(ring, tb, elem);
+  s.blk = o; o += align16(sizeof(int) * kSelectWarps * blocks_per_warp(tpc_max, tb));
   s.w = o; o += align16(sizeof(float) * tpc_max);
   s.r = o; o += align16(sizeof(float) * tpc_max);
   s.dl = o; o += align16(sizeof(float) * tpc_max);
@@ -176,9 +189,11 @@ select_kernel(const SelectArgs a) {
   const int voff = m[kVisOff], N = m[kNumVis], koff = m[kKeepOff], K = m[kNumKeep];
   if (K == 0) return;  // the whole cluster leaves together; no DSMEM traffic yet
 
-  const SelectSmem S = select_smem(a.cache_rows, a.row_bytes, a.tpc_max);
+  const SelectSmem S = select_smem(a.cache_rows, a.row_bytes, a.tpc_max, a.ring, TB, (int)sizeof(T));
   char *xcache = reinterpret_cast<char *>(smem + S.xcache);
   char *cbuf = reinterpret_cast<char *>(smem + S.cbuf);
+  const uint32_t ring_base = smem_addr(smem + S.ring);
+  int *blk_s = reinterpret_cast<int *>(smem + S.blk);
   float *w_s = reinterpret_cast<float *>(smem + S.w);
   float *r_s = reinterpret_cast<float *>(smem + S.r);
   float *dl_s = reinterpret_cast<float *>(smem + S.dl);
@@ -319,100 +334,148 @@ select_kernel(const SelectArgs a) {
     // centre 0 and are ignored) so that the independent chains interleave.
     auto update_nb = [&](auto nb_tag, int nA) {
       constexpr int NB = decltype(nb_tag)::value;
-      constexpr int NP = NB / 2;   // centre pairs: one __ffma2_rn serves two centres
+      constexpr int NP = NB / 2;   // centre pairs: one __ffma2_rn serves two centres (fp32)
+      (void)NP;
       constexpr int V = Elem<T>::kPerVec;
       constexpr int VPG = 8 / V;   // 16-byte vectors per 8-coordinate group
       int coff[NB];
 #pragma unroll
       for (int c = 0; c < NB; ++c) coff[c] = lp_row[acc_s[c < nA ? c : 0]] * rb;
+      // this warp's token blocks that still hold an unselected token
+      int *blist = blk_s + warp * blocks_per_warp(a.tpc_max, TB);
+      int nact = 0;
+      for (int k0 = 0; (warp + k0 * kSelectWarps) * TB < nloc; k0 += 32) {
+        const int t0 = (warp + (k0 + lane) * kSelectWarps) * TB;
+        bool act = false;
+        if (t0 < nloc) {
+#pragma unroll
+          for (int q = 0; q < TB; ++q) act |= t0 + q < nloc && !sel_s[t0 + q];
+        }
+        const unsigned m = __ballot_sync(0xffffffffu, act);
+        if (act) blist[nact + __popc(m & ((1u << lane) - 1u))] = t0;
+        nact += __popc(m);
+      }
+      __syncwarp();
+      // Items (block j, group g) flow through a per-lane ring: each lane copies its own
+      // 16-byte pieces of the streamed rows kRing-1 items ahead and reads back only what
+      // it copied, so the ring needs no cross-lane synchronisation.
+      const int total = nact * NCH;
+      const uint32_t wring = ring_base + (uint32_t)(warp * kRing * TB * VPG * 512);
+      auto ring_addr = [&](int slot, int q, int h) {
+        return wring + (uint32_t)((((slot * TB + q) * VPG + h) * 32 + lane) * 16);
+      };
+      auto issue = [&](int i) {
+        if (i < total) {
+          const int j = i / NCH, g = i - j * NCH;
+          const int t0 = blist[j];
+          const int col = 256 * g + 8 * lane;
+          if (col < dv) {
+#pragma unroll
+            for (int q = 0; q < TB; ++q) {
+              const int tq = t0 + q;
+              if (tq < nloc && tq >= ncache) {
+#pragma unroll
+                for (int h = 0; h < VPG; ++h)
+                  cp_async16(ring_addr(i % kRing, q, h),
+                             xg + (long long)tq * rb + col * (int)sizeof(T) + 16 * h);
+              }
+            }
+          }
+        }
+        cp_async_commit();
+      };
+      for (int i = 0; i < kRing - 1; ++i) issue(i);
       TopList tl;
       tl.clear();
-      for (int t0 = warp * TB; t0 < nloc; t0 += kSelectWarps * TB) {
-        bool valid[TB];
-        bool any = false;
-#pragma unroll
-        for (int q = 0; q < TB; ++q) {
-          valid[q] = t0 + q < nloc && !sel_s[t0 + q];
-          any |= valid[q];
-        }
-        if (!any) continue;
-        const char *row[TB];
-        bool sh[TB];
-#pragma unroll
-        for (int q = 0; q < TB; ++q) {
-          const int tq = t0 + q < nloc ? t0 + q : t0;
-          sh[q] = tq < ncache;
-          row[q] = sh[q] ? xcache + (long long)tq * rb : xg + (long long)tq * rb;
-        }
-        float2 acc[TB][NP];   // .x: centre 2p, .y: centre 2p+1
-#pragma unroll
-        for (int q = 0; q < TB; ++q)
-#pragma unroll
-          for (int p = 0; p < NP; ++p) acc[q][p] = make_float2(0.f, 0.f);
-        U4 nxt[TB][VPG];
-        const int col0 = 8 * lane;
-        if (col0 < dv) {
+      float acc[TB][NB];
+      for (int i = 0; i < total; ++i) {
+        issue(i + kRing - 1);
+        cp_async_wait<kRing - 1>();
+        const int j = i / NCH, g = i - j * NCH;
+        const int t0 = blist[j];
+        if (g == 0) {
 #pragma unroll
           for (int q = 0; q < TB; ++q)
 #pragma unroll
-            for (int h = 0; h < VPG; ++h)
-              nxt[q][h] = sh[q] ? lds(row[q] + col0 * sizeof(T) + 16 * h)
-                                : ldg(row[q] + col0 * sizeof(T) + 16 * h);
+            for (int c = 0; c < NB; ++c) acc[q][c] = 0.f;
         }
-#pragma unroll 1
-        for (int g = 0; g < NCH; ++g) {
-          const int col = 256 * g + 8 * lane;
-          if (col >= dv) break;
-          float2 td[TB][8];   // token values, duplicated for the paired fma
+        const int col = 256 * g + 8 * lane;
+        if (col < dv) {
+          U4 cur[TB][VPG];
 #pragma unroll
           for (int q = 0; q < TB; ++q) {
-            float e8[8];
+            const int tq = t0 + q < nloc ? t0 + q : t0;   // padding slots reuse a real row
 #pragma unroll
-            for (int h = 0; h < VPG; ++h) Elem<T>::widen(nxt[q][h], e8 + h * V);
-#pragma unroll
-            for (int e = 0; e < 8; ++e) td[q][e] = make_float2(e8[e], e8[e]);
+            for (int h = 0; h < VPG; ++h)
+              cur[q][h] = tq < ncache ? lds(xcache + (long long)tq * rb + col * sizeof(T) + 16 * h)
+                                      : lds32(ring_addr(i % kRing, tq - t0, h));
           }
-          const int coln = col + 256;
-          if (g + 1 < NCH && coln < dv) {   // prefetch the next group of every token
+          // bf16: one mixed-precision fma per coordinate straight from the packed words;
+          // fp32: paired fmas over two centres.  Both follow the canonical order.
+          if constexpr (sizeof(T) == 2) {
+#pragma unroll
+            for (int c = 0; c < NB; ++c) {
+              const U4 cv = lds(cbuf + coff[c] + col * 2);
+              const uint32_t cw[4] = {cv.x, cv.y, cv.z, cv.w};
+#pragma unroll
+              for (int hw = 0; hw < 4; ++hw) {
+#pragma unroll
+                for (int q = 0; q < TB; ++q) {
+                  const uint32_t tw = hw == 0 ? cur[q][0].x : hw == 1 ? cur[q][0].y
+                                    : hw == 2 ? cur[q][0].z : cur[q][0].w;
+                  acc[q][c] = fma_bf16_lo(tw, cw[hw], acc[q][c]);
+                  acc[q][c] = fma_bf16_hi(tw, cw[hw], acc[q][c]);
+                }
+              }
+            }
+          } else {
+            float tk[TB][8];
 #pragma unroll
             for (int q = 0; q < TB; ++q)
 #pragma unroll
-              for (int h = 0; h < VPG; ++h)
-                nxt[q][h] = sh[q] ? lds(row[q] + coln * sizeof(T) + 16 * h)
-                                  : ldg(row[q] + coln * sizeof(T) + 16 * h);
-          }
+              for (int h = 0; h < VPG; ++h) Elem<T>::widen(cur[q][h], tk[q] + h * V);
 #pragma unroll
-          for (int p = 0; p < NP; ++p) {
-            float c0[8], c1[8];
-            load8<T, true>(cbuf + coff[2 * p], col, c0);
-            load8<T, true>(cbuf + coff[2 * p + 1], col, c1);
+            for (int p = 0; p < NP; ++p) {
+              float c0[8], c1[8];
+              load8<T, true>(cbuf + coff[2 * p], col, c0);
+              load8<T, true>(cbuf + coff[2 * p + 1], col, c1);
 #pragma unroll
-            for (int e = 0; e < 8; ++e) {
-              const float2 cc = make_float2(c0[e], c1[e]);
+              for (int e = 0; e < 8; ++e) {
+                const float2 cc = make_float2(c0[e], c1[e]);
 #pragma unroll
-              for (int q = 0; q < TB; ++q) acc[q][p] = __ffma2_rn(td[q][e], cc, acc[q][p]);
+                for (int q = 0; q < TB; ++q) {
+                  const float2 r2 = __ffma2_rn(make_float2(tk[q][e], tk[q][e]), cc,
+                                               make_float2(acc[q][2 * p], acc[q][2 * p + 1]));
+                  acc[q][2 * p] = r2.x;
+                  acc[q][2 * p + 1] = r2.y;
+                }
+              }
             }
           }
         }
+        if (g == NCH - 1) {
 #pragma unroll
-        for (int q = 0; q < TB; ++q) {
-          float dl = valid[q] ? dl_s[t0 + q] : 0.f;
-          const float ri = valid[q] ? r_s[t0 + q] : 0.f;
+          for (int q = 0; q < TB; ++q) {
+            const bool valid = t0 + q < nloc && !sel_s[t0 + q];
+            float dl = valid ? dl_s[t0 + q] : 0.f;
+            const float ri = valid ? r_s[t0 + q] : 0.f;
 #pragma unroll
-          for (int c = 0; c < NB; ++c) {
-            const float dot = butterfly_sum((c & 1) ? acc[q][c / 2].y : acc[q][c / 2].x);
-            if (c < nA) {
-              const float rc = lp_f[acc_s[c] * 3 + 2];
-              dl = fminf(dl, __fsub_rn(1.0f, __fmul_rn(__fmul_rn(dot, ri), rc)));
+            for (int c = 0; c < NB; ++c) {
+              const float dot = butterfly_sum(acc[q][c]);
+              if (c < nA) {
+                const float rc = lp_f[acc_s[c] * 3 + 2];
+                dl = fminf(dl, __fsub_rn(1.0f, __fmul_rn(__fmul_rn(dot, ri), rc)));
+              }
             }
-          }
-          if (valid[q]) {
-            const int tq = t0 + q;
-            if (lane == 0) dl_s[tq] = dl;
-            tl.insert(argmax_key(__fmul_rn(w_s[tq], dl), lo + tq));
+            if (valid) {
+              const int tq = t0 + q;
+              if (lane == 0) dl_s[tq] = dl;
+              tl.insert(argmax_key(__fmul_rn(w_s[tq], dl), lo + tq));
+            }
           }
         }
       }
+      cp_async_wait<0>();
       if (lane == 0) {
 #pragma unroll
         for (int i = 0; i < kTopM; ++i) wtop[warp * kTopM + i] = tl.k[i];
@@ -728,6 +791,13 @@ cudaError_t launch_select(const Plan &pl, const float *w, const void *x, int32_t
   };
   void *fn = pick(4);   // sizes the cluster; both block widths have the same footprint
   const int optin = device_smem_optin();
+  double l2 = 0.0;
+  {
+    int dev = 0, v = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&v, cudaDevAttrL2CacheSize, dev);
+    l2 = v;
+  }
   cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   if (e != cudaSuccess) return e;
   // Cluster size: every cluster size the device can place is costed as
@@ -737,12 +807,22 @@ cudaError_t launch_select(const Plan &pl, const float *w, const void *x, int32_t
   int C = 0, tpc = 0, cache_rows = 0;
   size_t smem = 0;
   double best = 0.0;
+  int ring = 0;
   for (int c = 1; c <= kMaxCluster; c *= 2) {
     const int tpc_c = (pl.max_vis + c - 1) / c;
-    const size_t fixed = select_smem(0, rb, tpc_c).total;
-    if (fixed > (size_t)optin) continue;
-    const int cache_c = (int)std::min<size_t>(tpc_c, (optin - fixed) / rb);
-    const size_t smem_c = select_smem(cache_c, rb, tpc_c).total;
+    const int tb_c = (pl.elem == 4 || tpc_c < 64) ? 2 : 4;
+    // rows that fit without a ring; otherwise reserve the ring and cache what is left
+    const size_t fixed0 = select_smem(0, rb, tpc_c, 0, tb_c, pl.elem).total;
+    if (fixed0 > (size_t)optin) continue;
+    int ring_c = 0;
+    int cache_c = (int)std::min<size_t>(tpc_c, (optin - fixed0) / rb);
+    if (cache_c < tpc_c) {
+      ring_c = 1;
+      const size_t fixed1 = select_smem(0, rb, tpc_c, 1, tb_c, pl.elem).total;
+      if (fixed1 > (size_t)optin) continue;
+      cache_c = (int)std::min<size_t>(tpc_c, (optin - fixed1) / rb);
+    }
+    const size_t smem_c = select_smem(cache_c, rb, tpc_c, ring_c, tb_c, pl.elem).total;
     e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_c);
     if (e != cudaSuccess) return e;
     cudaLaunchConfig_t q = {};
@@ -762,16 +842,22 @@ cudaError_t launch_select(const Plan &pl, const float *w, const void *x, int32_t
       continue;
     }
     const double waves = std::ceil((double)pl.B / active);
-    const double round_cycles = (double)tpc_c * pl.dv * 8.0 / 96.0 + 9000.0 + 400.0 * c;
+    // features of the requests in flight beyond L2 stream from HBM (about 3x slower
+    // per row than from L2 or shared memory)
+    const double in_flight = std::min<double>(pl.B, active) * pl.max_vis * (double)rb;
+    const double stream_penalty = in_flight > 0.7 * l2 ? 3.0 : 1.0;
+    const double streamed = std::max(0, tpc_c - cache_c), cached = std::min(tpc_c, cache_c);
+    const double round_cycles =
+        (cached + stream_penalty * streamed) * pl.dv * 8.0 / 56.0 + 16000.0 + 400.0 * c;
     const double cost = waves * round_cycles;
     if (C == 0 || cost < best) {
-      best = cost; C = c; tpc = tpc_c; cache_rows = cache_c; smem = smem_c;
+      best = cost; C = c; tpc = tpc_c; cache_rows = cache_c; smem = smem_c; ring = ring_c;
     }
   }
   if (C == 0) return cudaErrorInvalidConfiguration;
   // 4-token register blocks amortise the centre loads best; 2-token blocks balance
   // the warps better when a CTA owns few tokens
-  fn = pick(tpc >= 64 ? 4 : 2);
+  fn = pick(pl.elem == 4 || tpc < 64 ? 2 : 4);
   e = cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   if (e != cudaSuccess) return e;
   e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
@@ -783,7 +869,8 @@ cudaError_t launch_select(const Plan &pl, const float *w, const void *x, int32_t
   a.order = reinterpret_cast<const int32_t *>(ws + pl.off_order);
   a.dv = pl.dv; a.row_bytes = rb; a.tpc_max = tpc; a.cache_rows = cache_rows; a.csize = C;
   // enough candidates per CTA that the list approximates the global top 16
-  a.mc = std::min(kTopM - 1, std::max(4, kLcap / C));
+  a.mc = C <= 4 ? kTopM - 1 : 4;
+  a.ring = ring;
   a.err = reinterpret_cast<unsigned *>(ws + pl.off_err);
 
   cudaLaunchConfig_t cfg = {};
