@@ -41,7 +41,7 @@ FP32_LANES_PER_SM = 128
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=300)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--budget", default="mixed", help="c2 budget: mixed, 64, 128 or 192")
@@ -87,7 +87,7 @@ def score_bytes(wl):
 
 
 class ClockSampler:
-    """nvidia-smi clocks/throttle reasons sampled every 200 ms while running."""
+    """nvidia-smi clocks/throttle reasons sampled every 100 ms while running."""
 
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
@@ -104,7 +104,7 @@ class ClockSampler:
             os.close(fd)
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
-                 "--format=csv,noheader,nounits", "-lms", "200"],
+                 "--format=csv,noheader,nounits", "-lms", "100"],
                 stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
             time.sleep(0.3)
         except (OSError, FileNotFoundError):
@@ -145,6 +145,37 @@ class ClockSampler:
         return {"sm_mhz": statistics.median(r["sm"] for r in loaded),
                 "sm_max_mhz": max(r["smax"] for r in rows), "reasons": sorted(reasons),
                 "samples": len(rows), "power_w_max": max(r["power"] for r in rows)}
+
+
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "select_kernel_traffic.txt")
+
+
+def measured_traffic(kernel_source: str, workload: str):
+    """DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) recorded
+    from an ncu capture of this workload, or None when the kernel source has changed
+    since (its SHA-256 no longer matches the one recorded with the counters).
+    The record is `key value` lines; a `workload` line starts each entry."""
+    import hashlib
+    rec, cur = {}, None
+    try:
+        with open(TRAFFIC_FILE) as f:
+            for line in f:
+                parts = line.split()
+                if len(parts) != 2 or line.startswith("#"):
+                    continue
+                if parts[0] == "workload":
+                    cur = rec.setdefault(parts[1], {})
+                elif cur is not None:
+                    cur[parts[0]] = parts[1]
+        src = os.path.join(ROOT, "paper_2607_27952_gb300", "csrc", kernel_source)
+        with open(src, "rb") as f:
+            digest = hashlib.sha256(f.read()).hexdigest()
+    except OSError:
+        return None
+    r = rec.get(workload)
+    if not r or r.get("source_sha256") != digest or "dram_bytes_per_launch" not in r:
+        return None
+    return int(r["dram_bytes_per_launch"])
 
 
 def peaks():
@@ -320,7 +351,7 @@ def main():
                     "scores_GBps": sc_gbs, "scores_hbm_frac": sc_gbs / hbm},
         "roofline": {"bound": "alu", "kernel": "select_kernel", "achieved": achieved,
                      "peak": alu_peak_tflops, "unit": "TFLOP/s", "frac": achieved / alu_peak_tflops,
-                     "traffic": None,
+                     "traffic": measured_traffic("select_kernels.cu", f"c2-{args.budget}"),
                      "peak_note": f"{sm_count} SMs x {FP32_LANES_PER_SM} fp32 FMA/clk x 2 x "
                                   f"{sm_max:.0f} MHz ({pk_kind} max clock)"},
         "clocks": clocks,

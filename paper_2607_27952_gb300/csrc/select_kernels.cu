@@ -44,7 +44,8 @@ namespace last {
 
 constexpr int kSelThreads = kSelectWarps * 32;
 constexpr int kMaxCluster = 16;
-constexpr int kLcap = 16;                          // candidate list length
+constexpr int kLcap = 32;                          // candidate list capacity (runtime a.lcap <= kLcap)
+constexpr int kMaxAccept = 16;                     // picks folded into delta per round
 constexpr int kTopM = 9;                           // per-warp / per-CTA ranked keys (<= 8 + bound)
 constexpr int kMaxPairs = kLcap * (kLcap - 1) / 2;
 constexpr int kRing = 4;                           // async-copy ring depth (groups in flight)
@@ -59,6 +60,7 @@ struct SelectArgs {
   int dv, row_bytes, tpc_max, cache_rows, csize;
   int mc;                // candidates each CTA publishes per round (<= kTopM - 1)
   int ring;              // 1: rows beyond the resident cache stream through an async-copy ring
+  int lcap;              // candidate list length (16 or 32)
   unsigned *err;         // workspace error word
 };
 
@@ -77,11 +79,11 @@ __host__ __device__ inline int blocks_per_warp(int tpc_max, int tb) {
   return (tpc_max + kSelectWarps * tb - 1) / (kSelectWarps * tb);
 }
 __host__ __device__ inline SelectSmem select_smem(int cache_rows, int row_bytes, int tpc_max,
-                                                  int ring, int tb, int elem) {
+                                                  int ring, int tb, int elem, int lcap) {
   SelectSmem s;
   size_t o = 0;
   s.xcache = o; o += (size_t)cache_rows * row_bytes;
-  s.cbuf = o; o += (size_t)kLcap * row_bytes;
+  s.cbuf = o; o += (size_t)lcap * row_bytes;
   s.ring = o; o += ring_bytes(ring, tb, elem);
   s.blk = o; o += align16(sizeof(int) * kSelectWarps * blocks_per_warp(tpc_max, tb));
   s.w = o; o += align16(sizeof(float) * tpc_max);
@@ -97,7 +99,7 @@ __host__ __device__ inline SelectSmem select_smem(int cache_rows, int row_bytes,
   s.lp_idx = o; o += sizeof(int) * kLcap;
   s.lp_row = o; o += sizeof(int) * kLcap;
   s.pair = o; o += sizeof(float) * 2 * kMaxPairs;
-  s.acc = o; o += sizeof(int) * kLcap;
+  s.acc = o; o += sizeof(int) * kMaxAccept;
   s.misc = o; o += sizeof(unsigned long long) * (4 + kTopM);
   s.bar = o; o += sizeof(unsigned long long);
   s.cnt = o; o += sizeof(int) * kMaxCluster;
@@ -189,7 +191,9 @@ select_kernel(const SelectArgs a) {
   const int voff = m[kVisOff], N = m[kNumVis], koff = m[kKeepOff], K = m[kNumKeep];
   if (K == 0) return;  // the whole cluster leaves together; no DSMEM traffic yet
 
-  const SelectSmem S = select_smem(a.cache_rows, a.row_bytes, a.tpc_max, a.ring, TB, (int)sizeof(T));
+  const SelectSmem S = select_smem(a.cache_rows, a.row_bytes, a.tpc_max, a.ring, TB, (int)sizeof(T),
+                                   a.lcap);
+  const int lcap = a.lcap;
   char *xcache = reinterpret_cast<char *>(smem + S.xcache);
   char *cbuf = reinterpret_cast<char *>(smem + S.cbuf);
   const uint32_t ring_base = smem_addr(smem + S.ring);
@@ -323,7 +327,7 @@ select_kernel(const SelectArgs a) {
     // With few CTAs every published candidate fits in cbuf: copy them all right after
     // the exchange (published entry e of CTA q -> cbuf row q * mc + e), overlapping the
     // copies with the list construction.
-    const bool early = C * a.mc <= kLcap;
+    const bool early = C * a.mc <= lcap;
 
     // delta_i <- min(delta_i, 1 - (dot(x_i, x_c) r_i) r_c) over the nA accepted
     // centres (cbuf rows acc_s[0..nA)), for every unselected local token; then the
@@ -358,120 +362,131 @@ select_kernel(const SelectArgs a) {
       __syncwarp();
       // Items (block j, group g) flow through a per-lane ring: each lane copies its own
       // 16-byte pieces of the streamed rows kRing-1 items ahead and reads back only what
-      // it copied, so the ring needs no cross-lane synchronisation.
-      const int total = nact * NCH;
-      const uint32_t wring = ring_base + (uint32_t)(warp * kRing * TB * VPG * 512);
-      auto ring_addr = [&](int slot, int q, int h) {
-        return wring + (uint32_t)((((slot * TB + q) * VPG + h) * 32 + lane) * 16);
-      };
-      auto issue = [&](int i) {
-        if (i < total) {
-          const int j = i / NCH, g = i - j * NCH;
-          const int t0 = blist[j];
-          const int col = 256 * g + 8 * lane;
+      // it copied, so the ring needs no cross-lane synchronisation.  Fully resident
+      // blocks issue nothing.
+      const uint32_t wring = ring_base + (uint32_t)(warp * kRing * TB * VPG * 512) + lane * 16;
+      const uint32_t xc_base = smem_addr(xcache) + lane * 8 * (int)sizeof(T);
+      const uint32_t cb_base = smem_addr(cbuf) + lane * (int)sizeof(T) * 8;
+      const bool streams = a.ring && ncache < nloc;
+      int ij = 0, ig = 0;       // issue cursor: block, group
+      uint32_t islot = 0;       // ring slot of the next issue
+      auto issue = [&]() {
+        if (streams && ij < nact) {
+          const int t0 = blist[ij];
+          const int col = 256 * ig + 8 * lane;
           if (col < dv) {
+            const char *src = xg + (long long)t0 * rb + col * (int)sizeof(T);
 #pragma unroll
-            for (int q = 0; q < TB; ++q) {
-              const int tq = t0 + q;
-              if (tq < nloc && tq >= ncache) {
+            for (int q = 0; q < TB; ++q)
+              if (t0 + q < nloc && t0 + q >= ncache)
 #pragma unroll
                 for (int h = 0; h < VPG; ++h)
-                  cp_async16(ring_addr(i % kRing, q, h),
-                             xg + (long long)tq * rb + col * (int)sizeof(T) + 16 * h);
-              }
-            }
+                  cp_async16(wring + (islot * TB * VPG + q * VPG + h) * 512, src + (long long)q * rb + 16 * h);
           }
+          if (++ig == NCH) { ig = 0; ++ij; }
         }
+        islot = (islot + 1) & (kRing - 1);
         cp_async_commit();
       };
-      for (int i = 0; i < kRing - 1; ++i) issue(i);
+      if (streams)
+        for (int i = 0; i < kRing - 1; ++i) issue();
       TopList tl;
       tl.clear();
-      float acc[TB][NB];
-      for (int i = 0; i < total; ++i) {
-        issue(i + kRing - 1);
-        cp_async_wait<kRing - 1>();
-        const int j = i / NCH, g = i - j * NCH;
+      uint32_t cslot = 0;       // ring slot of the item being computed
+      for (int j = 0; j < nact; ++j) {
         const int t0 = blist[j];
-        if (g == 0) {
+        uint32_t tok[TB];       // per-token shared address of group 0 (resident) or ring base
+        bool res[TB];
 #pragma unroll
-          for (int q = 0; q < TB; ++q)
-#pragma unroll
-            for (int c = 0; c < NB; ++c) acc[q][c] = 0.f;
+        for (int q = 0; q < TB; ++q) {
+          const int tq = t0 + q < nloc ? t0 + q : t0;   // padding slots reuse a real row
+          res[q] = tq < ncache;
+          tok[q] = res[q] ? xc_base + (uint32_t)(tq * rb) : wring + (uint32_t)((tq - t0) * VPG * 512);
         }
-        const int col = 256 * g + 8 * lane;
-        if (col < dv) {
-          U4 cur[TB][VPG];
+        float acc[TB][NB];
 #pragma unroll
-          for (int q = 0; q < TB; ++q) {
-            const int tq = t0 + q < nloc ? t0 + q : t0;   // padding slots reuse a real row
+        for (int q = 0; q < TB; ++q)
 #pragma unroll
-            for (int h = 0; h < VPG; ++h)
-              cur[q][h] = tq < ncache ? lds(xcache + (long long)tq * rb + col * sizeof(T) + 16 * h)
-                                      : lds32(ring_addr(i % kRing, tq - t0, h));
+          for (int c = 0; c < NB; ++c) acc[q][c] = 0.f;
+#pragma unroll 1
+        for (int g = 0; g < NCH; ++g) {
+          if (streams) {
+            issue();
+            cp_async_wait<kRing - 1>();
           }
-          // bf16: one mixed-precision fma per coordinate straight from the packed words;
-          // fp32: paired fmas over two centres.  Both follow the canonical order.
-          if constexpr (sizeof(T) == 2) {
-#pragma unroll
-            for (int c = 0; c < NB; ++c) {
-              const U4 cv = lds(cbuf + coff[c] + col * 2);
-              const uint32_t cw[4] = {cv.x, cv.y, cv.z, cv.w};
-#pragma unroll
-              for (int hw = 0; hw < 4; ++hw) {
-#pragma unroll
-                for (int q = 0; q < TB; ++q) {
-                  const uint32_t tw = hw == 0 ? cur[q][0].x : hw == 1 ? cur[q][0].y
-                                    : hw == 2 ? cur[q][0].z : cur[q][0].w;
-                  acc[q][c] = fma_bf16_lo(tw, cw[hw], acc[q][c]);
-                  acc[q][c] = fma_bf16_hi(tw, cw[hw], acc[q][c]);
-                }
-              }
-            }
-          } else {
-            float tk[TB][8];
+          if (256 * g + 8 * lane < dv) {
+            U4 cur[TB][VPG];
 #pragma unroll
             for (int q = 0; q < TB; ++q)
 #pragma unroll
-              for (int h = 0; h < VPG; ++h) Elem<T>::widen(cur[q][h], tk[q] + h * V);
+              for (int h = 0; h < VPG; ++h)
+                cur[q][h] = lds32(res[q] ? tok[q] + (uint32_t)(g * 8 * sizeof(T) * 32 + 16 * h)
+                                         : tok[q] + (uint32_t)((cslot * TB * VPG + h) * 512));
+            const uint32_t cg = cb_base + (uint32_t)(g * 8 * sizeof(T) * 32);
+            // bf16: one mixed-precision fma per coordinate straight from the packed words;
+            // fp32: paired fmas over two centres.  Both follow the canonical order.
+            if constexpr (sizeof(T) == 2) {
 #pragma unroll
-            for (int p = 0; p < NP; ++p) {
-              float c0[8], c1[8];
-              load8<T, true>(cbuf + coff[2 * p], col, c0);
-              load8<T, true>(cbuf + coff[2 * p + 1], col, c1);
+              for (int c = 0; c < NB; ++c) {
+                const U4 cv = lds32(cg + (uint32_t)coff[c]);
+                const uint32_t cw[4] = {cv.x, cv.y, cv.z, cv.w};
 #pragma unroll
-              for (int e = 0; e < 8; ++e) {
-                const float2 cc = make_float2(c0[e], c1[e]);
+                for (int hw = 0; hw < 4; ++hw) {
 #pragma unroll
-                for (int q = 0; q < TB; ++q) {
-                  const float2 r2 = __ffma2_rn(make_float2(tk[q][e], tk[q][e]), cc,
-                                               make_float2(acc[q][2 * p], acc[q][2 * p + 1]));
-                  acc[q][2 * p] = r2.x;
-                  acc[q][2 * p + 1] = r2.y;
+                  for (int q = 0; q < TB; ++q) {
+                    const uint32_t tw = hw == 0 ? cur[q][0].x : hw == 1 ? cur[q][0].y
+                                      : hw == 2 ? cur[q][0].z : cur[q][0].w;
+                    acc[q][c] = fma_bf16_lo(tw, cw[hw], acc[q][c]);
+                    acc[q][c] = fma_bf16_hi(tw, cw[hw], acc[q][c]);
+                  }
+                }
+              }
+            } else {
+              float tk[TB][8];
+#pragma unroll
+              for (int q = 0; q < TB; ++q)
+#pragma unroll
+                for (int h = 0; h < VPG; ++h) Elem<T>::widen(cur[q][h], tk[q] + h * V);
+#pragma unroll
+              for (int p = 0; p < NP; ++p) {
+                float c0[8], c1[8];
+                Elem<T>::widen(lds32(cg + (uint32_t)coff[2 * p]), c0);
+                Elem<T>::widen(lds32(cg + (uint32_t)coff[2 * p] + 16), c0 + 4);
+                Elem<T>::widen(lds32(cg + (uint32_t)coff[2 * p + 1]), c1);
+                Elem<T>::widen(lds32(cg + (uint32_t)coff[2 * p + 1] + 16), c1 + 4);
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                  const float2 cc = make_float2(c0[e], c1[e]);
+#pragma unroll
+                  for (int q = 0; q < TB; ++q) {
+                    const float2 r2 = __ffma2_rn(make_float2(tk[q][e], tk[q][e]), cc,
+                                                 make_float2(acc[q][2 * p], acc[q][2 * p + 1]));
+                    acc[q][2 * p] = r2.x;
+                    acc[q][2 * p + 1] = r2.y;
+                  }
                 }
               }
             }
           }
+          cslot = (cslot + 1) & (kRing - 1);
         }
-        if (g == NCH - 1) {
 #pragma unroll
-          for (int q = 0; q < TB; ++q) {
-            const bool valid = t0 + q < nloc && !sel_s[t0 + q];
-            float dl = valid ? dl_s[t0 + q] : 0.f;
-            const float ri = valid ? r_s[t0 + q] : 0.f;
+        for (int q = 0; q < TB; ++q) {
+          const bool valid = t0 + q < nloc && !sel_s[t0 + q];
+          float dl = valid ? dl_s[t0 + q] : 0.f;
+          const float ri = valid ? r_s[t0 + q] : 0.f;
 #pragma unroll
-            for (int c = 0; c < NB; ++c) {
+          for (int c = 0; c < NB; ++c) {
+            if (c < nA) {
               const float dot = butterfly_sum(acc[q][c]);
-              if (c < nA) {
-                const float rc = lp_f[acc_s[c] * 3 + 2];
-                dl = fminf(dl, __fsub_rn(1.0f, __fmul_rn(__fmul_rn(dot, ri), rc)));
-              }
+              const float rc = lp_f[acc_s[c] * 3 + 2];
+              dl = fminf(dl, __fsub_rn(1.0f, __fmul_rn(__fmul_rn(dot, ri), rc)));
             }
-            if (valid) {
-              const int tq = t0 + q;
-              if (lane == 0) dl_s[tq] = dl;
-              tl.insert(argmax_key(__fmul_rn(w_s[tq], dl), lo + tq));
-            }
+          }
+          if (valid) {
+            const int tq = t0 + q;
+            if (lane == 0) dl_s[tq] = dl;
+            tl.insert(argmax_key(__fmul_rn(w_s[tq], dl), lo + tq));
           }
         }
       }
@@ -538,7 +553,7 @@ select_kernel(const SelectArgs a) {
                        (uint32_t)rb, bar);
           }
       }
-      // candidate list: published top-mc entries above U, best first, at most kLcap
+      // candidate list: published top-mc entries above U, best first, at most lcap
       if (warp == 0) {
         const int kPer = a.mc;
         const int ne = C * kPer;
@@ -569,7 +584,7 @@ select_kernel(const SelectArgs a) {
         unsigned long long cut = 0ull;
         auto place = [&](bool cand, int pos, unsigned long long ke, int slot) {
           if (!cand) return;
-          if (pos < kLcap) {
+          if (pos < lcap) {
             const float4 f = pub_f[slot];
             lp_key[pos] = ke;
             lp_idx[pos] = key_index(ke);
@@ -577,7 +592,7 @@ select_kernel(const SelectArgs a) {
             lp_f[pos * 3 + 0] = f.x;
             lp_f[pos * 3 + 1] = f.y;
             lp_f[pos * 3 + 2] = f.z;
-          } else if (pos == kLcap) {
+          } else if (pos == lcap) {
             cut = ke;
           }
         };
@@ -591,7 +606,7 @@ select_kernel(const SelectArgs a) {
         }
         if (lane == 0) {
           misc[0] = cut > U ? cut : U;               // U' bounds everything outside L
-          misc[1] = (unsigned long long)min(ncand, kLcap);
+          misc[1] = (unsigned long long)min(ncand, lcap);
         }
       }
       __syncthreads();
@@ -647,7 +662,7 @@ select_kernel(const SelectArgs a) {
         const float rv = pending ? lp_f[lane * 3 + 2] : 0.f;
         const int gi = pending ? lp_idx[lane] : 0;
         int nA = 0;
-        while (taken + nA < K) {
+        while (taken + nA < K && nA < kMaxAccept) {
           // argmax of the pending keys: high word (ordered value) then low word (index)
           const uint32_t khi = pending ? (uint32_t)(key >> 32) : 0u;
           const uint32_t mhi = __reduce_max_sync(0xffffffffu, khi);
@@ -807,22 +822,23 @@ cudaError_t launch_select(const Plan &pl, const float *w, const void *x, int32_t
   int C = 0, tpc = 0, cache_rows = 0;
   size_t smem = 0;
   double best = 0.0;
-  int ring = 0;
+  int ring = 0, lcap = kLcap / 2;
   for (int c = 1; c <= kMaxCluster; c *= 2) {
     const int tpc_c = (pl.max_vis + c - 1) / c;
     const int tb_c = (pl.elem == 4 || tpc_c < 64) ? 2 : 4;
+    const int lcap_c = c <= 4 ? kLcap : kLcap / 2;
     // rows that fit without a ring; otherwise reserve the ring and cache what is left
-    const size_t fixed0 = select_smem(0, rb, tpc_c, 0, tb_c, pl.elem).total;
+    const size_t fixed0 = select_smem(0, rb, tpc_c, 0, tb_c, pl.elem, lcap_c).total;
     if (fixed0 > (size_t)optin) continue;
     int ring_c = 0;
     int cache_c = (int)std::min<size_t>(tpc_c, (optin - fixed0) / rb);
     if (cache_c < tpc_c) {
       ring_c = 1;
-      const size_t fixed1 = select_smem(0, rb, tpc_c, 1, tb_c, pl.elem).total;
+      const size_t fixed1 = select_smem(0, rb, tpc_c, 1, tb_c, pl.elem, lcap_c).total;
       if (fixed1 > (size_t)optin) continue;
       cache_c = (int)std::min<size_t>(tpc_c, (optin - fixed1) / rb);
     }
-    const size_t smem_c = select_smem(cache_c, rb, tpc_c, ring_c, tb_c, pl.elem).total;
+    const size_t smem_c = select_smem(cache_c, rb, tpc_c, ring_c, tb_c, pl.elem, lcap_c).total;
     e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_c);
     if (e != cudaSuccess) return e;
     cudaLaunchConfig_t q = {};
@@ -852,6 +868,7 @@ cudaError_t launch_select(const Plan &pl, const float *w, const void *x, int32_t
     const double cost = waves * round_cycles;
     if (C == 0 || cost < best) {
       best = cost; C = c; tpc = tpc_c; cache_rows = cache_c; smem = smem_c; ring = ring_c;
+      lcap = lcap_c;
     }
   }
   if (C == 0) return cudaErrorInvalidConfiguration;
@@ -871,6 +888,7 @@ cudaError_t launch_select(const Plan &pl, const float *w, const void *x, int32_t
   // enough candidates per CTA that the list approximates the global top 16
   a.mc = C <= 4 ? kTopM - 1 : 4;
   a.ring = ring;
+  a.lcap = lcap;
   a.err = reinterpret_cast<unsigned *>(ws + pl.off_err);
 
   cudaLaunchConfig_t cfg = {};
