@@ -45,28 +45,62 @@ def parse():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--budget", default="mixed", help="c2 budget: mixed, 64, 128 or 192")
+    ap.add_argument("--workload", default="c2", choices=["c1", "c2", "c3", "c4", "c5"],
+                    help="c2 (default) is the benchmark line; the others are reported for context")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     return ap.parse_args()
 
 
-def workload(budget, rank):
+def rank_seed(rank: int) -> int:
+    """Each rank prunes its own batch of independent requests (weak scaling)."""
+    return 1 + 1000 * rank
+
+
+def workload(budget, rank, name="c2"):
     from workloads import config
-    b = budget if budget == "mixed" else int(budget)
-    # each rank prunes its own batch (independent requests, weak scaling)
-    return config("c2", budget=b, seed=1 + 1000 * rank)
+    if name == "c2":
+        b = budget if budget == "mixed" else int(budget)
+        return config("c2", budget=b, seed=rank_seed(rank))
+    if name == "c5":
+        return config("c5", budget=12.5 if budget == "mixed" else float(budget),
+                      seed=4 + 1000 * rank)
+    base = {"c1": 0, "c3": 2, "c4": 3}[name]
+    return config(name, seed=base + 1000 * rank)
 
 
-def workload_desc(wl, budget):
+def combine_over_ranks(total_ms: float, requests: int, tokens: int, device=None):
+    """Whole-job figures: the slowest rank's time and the requests / visual tokens of
+    all ranks (replicas only: no data-path collective, just this reduction of
+    timings).  Returns (max_ms, total_requests, total_tokens)."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return total_ms, requests, tokens
+    t = torch.tensor([total_ms], dtype=torch.float64, device=device)
+    n = torch.tensor([requests, tokens], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    dist.all_reduce(n, op=dist.ReduceOp.SUM)
+    return float(t.item()), int(n[0].item()), int(n[1].item())
+
+
+def workload_desc(wl, budget, name="c2"):
     n = np.diff(wl.cu_vis)
     k = np.diff(wl.cu_keep)
-    return {"workload": f"c2: {wl.batch} requests x {int(n[0])} visual tokens (LLaVA-1.5 shape), "
-                        f"budgets {'64/128/192 round-robin' if budget == 'mixed' else budget}",
+    if name == "c2":
+        title = (f"c2: {wl.batch} requests x {int(n[0])} visual tokens (LLaVA-1.5 shape), "
+                 f"budgets {'64/128/192 round-robin' if budget == 'mixed' else budget}")
+    else:
+        title = f"{wl.name}: {wl.batch} requests, {wl.note}"
+    in_bytes = int(wl.q.nbytes + wl.k.nbytes + wl.x.nbytes)
+    return {"workload": title,
             "batch": wl.batch, "visual_tokens": int(n.sum()), "kept_tokens": int(k.sum()),
             "keys": int(wl.cu_seqlens[-1]), "layers": wl.num_layers, "q_heads": wl.num_q_heads,
             "kv_heads": wl.num_kv_heads, "head_dim": wl.head_dim, "feat_dim": wl.feat_dim,
-            "input_bytes": int(wl.q.nbytes + wl.k.nbytes + wl.x.nbytes),
-            "l2": "inputs (321 MB) larger than L2 (129 MB); no flush"}
+            "input_dtype": wl.dtype, "input_bytes": in_bytes,
+            "l2": (f"inputs ({in_bytes / 1e6:.0f} MB) larger than L2 (129 MB); no flush"
+                   if in_bytes > 129e6 else
+                   f"inputs ({in_bytes / 1e6:.1f} MB) fit in L2: steady-state, L2-warm figure")}
 
 
 def select_fmas(wl):
@@ -79,6 +113,19 @@ def select_fmas(wl):
         if 0 < k < n:
             tot += n + (k - 1) * n - k * (k - 1) // 2
     return tot * wl.feat_dim
+
+
+def prune_bytes_moved(wl):
+    """Bytes the fused prune moves under the accounting of its HBM-roofline target:
+    compulsory bytes (K, q and X read once, w~ written, X_S written and its rows
+    read) plus the greedy's own feature reads, k_b * N_b * d_v elements per request
+    (the O(K N d_v) distance work of Sec. 3.4), valued at HBM rate."""
+    e = wl.elem_bytes
+    keep = int(wl.cu_keep[-1])
+    comp = wl.k.nbytes + wl.q.nbytes + wl.x.nbytes + 4 * int(wl.cu_vis[-1]) + 2 * keep * wl.feat_dim * e
+    greedy = sum(int(wl.cu_keep[b + 1] - wl.cu_keep[b]) * int(wl.cu_vis[b + 1] - wl.cu_vis[b])
+                 for b in range(wl.batch)) * wl.feat_dim * e
+    return comp, greedy
 
 
 def score_bytes(wl):
@@ -270,20 +317,22 @@ def main():
         dist.init_process_group("nccl", device_id=dev)
     last.load_library()
 
-    wl = workload(args.budget, rank)
+    wl = workload(args.budget, rank, args.workload)
     prob = last.Problem(batch=wl.batch, num_layers=wl.num_layers, num_q_heads=wl.num_q_heads,
                         num_kv_heads=wl.num_kv_heads, head_dim=wl.head_dim, feat_dim=wl.feat_dim,
                         dtype=wl.dtype, cu_seqlens=wl.cu_seqlens, vis_start=wl.vis_start,
                         cu_vis=wl.cu_vis, cu_keep=wl.cu_keep)
 
     def dev_t(a):
-        return torch.from_numpy(a.view(np.int16)).to(dev).view(torch.bfloat16)
+        if a.dtype == np.uint16:
+            return torch.from_numpy(a.view(np.int16)).to(dev).view(torch.bfloat16)
+        return torch.from_numpy(a).to(dev)
 
     q, k, x = dev_t(wl.q), dev_t(wl.k), dev_t(wl.x)
     nvis, nkeep = int(wl.cu_vis[-1]), int(wl.cu_keep[-1])
     w = torch.empty(nvis, dtype=torch.float32, device=dev)
     idx = torch.empty(nkeep, dtype=torch.int32, device=dev)
-    xs = torch.empty((nkeep, wl.feat_dim), dtype=torch.bfloat16, device=dev)
+    xs = torch.empty((nkeep, wl.feat_dim), dtype=x.dtype, device=dev)
     ws = last.workspace(prob, dev)
     stream = torch.cuda.current_stream(dev)
 
@@ -317,14 +366,9 @@ def main():
     total_ms = ev[0][0].elapsed_time(ev[-1][2])
     scores_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in ev)
     select_ms = statistics.mean(e[1].elapsed_time(e[2]) for e in ev)
-    if world > 1:
-        t = torch.tensor([total_ms], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        total_ms = float(t.item())
-
-    reqs = wl.batch * world * K
+    total_ms, reqs, toks = combine_over_ranks(total_ms, wl.batch * K, nvis * K, device=dev)
     value = reqs / (total_ms / 1e3)
-    tokens_per_s = nvis * world * K / (total_ms / 1e3)
+    tokens_per_s = toks / (total_ms / 1e3)
 
     pk, pk_kind = peaks()
     sm_count = torch.cuda.get_device_properties(dev).multi_processor_count
@@ -339,12 +383,14 @@ def main():
     if not args.no_e2e:
         e2e = measure_e2e(args, wl, prob, dev, stream, last, q, k, x)
 
+    comp, greedy = prune_bytes_moved(wl)
+    moved_tbs = (comp + greedy) / (total_ms / K / 1e3) / 1e12
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
         "warmup": args.warmup, "ms_per_step": total_ms / K, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16 in, fp32 compute",
         "data": "synthetic (seeded; shapes of the paper's LLaVA-1.5 workload)",
-        "config": workload_desc(wl, args.budget) | {"parallelism": f"replicas x{world}"},
+        "config": workload_desc(wl, args.budget, args.workload) | {"parallelism": f"replicas x{world}"},
         "visual_tokens_scored_per_s": tokens_per_s,
         "gpu_launches": 3 * K,
         "kernels": {"scores_ms": scores_ms, "select_ms": select_ms,
@@ -355,6 +401,11 @@ def main():
                      "peak_note": f"{sm_count} SMs x {FP32_LANES_PER_SM} fp32 FMA/clk x 2 x "
                                   f"{sm_max:.0f} MHz ({pk_kind} max clock)"},
         "clocks": clocks,
+        "prune_bytes_moved": {"compulsory_bytes": comp, "greedy_feature_bytes": greedy,
+                              "achieved_TBps": moved_tbs, "hbm_peak_TBps": hbm / 1e3,
+                              "frac": moved_tbs / (hbm / 1e3),
+                              "note": "bytes-moved accounting of the 70% HBM target; the greedy "
+                                      "reads are served from shared memory / L2"},
     }
     if e2e is not None:
         line["e2e"] = e2e
@@ -371,13 +422,16 @@ def measure_e2e(args, wl, prob, dev, stream, last, q_d, k_d, x_d):
     copies q, K, X from pinned host memory, prunes, and reads back the kept indices and
     rows."""
     import torch
-    pin = lambda a: torch.from_numpy(a.view(np.int16)).view(torch.bfloat16).pin_memory()
+    def pin(a):
+        if a.dtype == np.uint16:
+            return torch.from_numpy(a.view(np.int16)).view(torch.bfloat16).pin_memory()
+        return torch.from_numpy(a).pin_memory()
     qh, kh, xh = pin(wl.q), pin(wl.k), pin(wl.x)
     nkeep = int(wl.cu_keep[-1])
     idx_h = torch.empty(nkeep, dtype=torch.int32).pin_memory()
-    xs_h = torch.empty((nkeep, wl.feat_dim), dtype=torch.bfloat16).pin_memory()
+    xs_h = torch.empty((nkeep, wl.feat_dim), dtype=xh.dtype).pin_memory()
     idx_d = torch.empty(nkeep, dtype=torch.int32, device=dev)
-    xs_d = torch.empty((nkeep, wl.feat_dim), dtype=torch.bfloat16, device=dev)
+    xs_d = torch.empty((nkeep, wl.feat_dim), dtype=xh.dtype, device=dev)
     ws = last.workspace(prob, dev)
 
     def step():
@@ -399,8 +453,8 @@ def measure_e2e(args, wl, prob, dev, stream, last, q_d, k_d, x_d):
     e1.record(stream)
     torch.cuda.synchronize(dev)
     ms = e0.elapsed_time(e1)
-    h2d = int(qh.numel() + kh.numel() + xh.numel()) * 2
-    d2h = int(idx_h.numel() * 4 + xs_h.numel() * 2)
+    h2d = int(qh.numel() + kh.numel() + xh.numel()) * xh.element_size()
+    d2h = int(idx_h.numel() * 4 + xs_h.numel() * xs_h.element_size())
     return {"value": wl.batch * steps / (ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "steps": steps}
 

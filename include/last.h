@@ -47,11 +47,10 @@
  *   q-head h reads kv-head h / (num_q_heads / num_kv_heads).
  *
  * Limits (LAST_ERR_UNSUPPORTED beyond them; last_error_message() says which):
- *   scoring   G = num_q_heads / num_kv_heads in 1..8; head_dim * elem_bytes is
- *             16 bytes times a power of two, at most 512 bytes (1024 when G <= 2);
- *             num_kv_heads * head_dim * elem_bytes small enough that one key's
- *             row fits one 256-thread CTA pass (e.g. 16 x 128 bf16, 16 x 64 fp32);
- *             num_layers * num_q_heads <= 6144.
+ *   scoring   G = num_q_heads / num_kv_heads in 1..8; head_dim * elem_bytes a
+ *             multiple of 16; num_q_heads * head_dim fp32 values of q plus one
+ *             chunk of logits within 100 KB of shared memory (e.g. up to 128
+ *             q-heads of 128); num_layers * num_q_heads <= 6144.
  *   selection feat_dim a multiple of 8, at most 2048.
  */
 #ifndef LAST_H_

@@ -79,6 +79,7 @@ last_status make_plan(const last_problem *p, bool need_scores, bool need_select,
       return fail(LAST_ERR_UNSUPPORTED, "num_layers * num_q_heads must be <= 6144");
     if (p->cu_seqlens[0] != 0) return fail(LAST_ERR_INVALID_ARG, "cu_seqlens[0] must be 0");
     pl->G = p->num_q_heads / p->num_kv_heads;
+    pl->chunk = score_chunk_keys(p->num_kv_heads);
     pl->scale = p->softmax_scale > 0.f ? p->softmax_scale
                                        : (float)(1.0 / std::sqrt((double)p->head_dim));
     for (int b = 0; b < B; ++b) {
@@ -91,7 +92,7 @@ last_status make_plan(const last_problem *p, bool need_scores, bool need_select,
         return fail(LAST_ERR_INVALID_ARG, "request " + std::to_string(b) +
                                               ": visual span must end before the query position");
       pl->max_seq = std::max(pl->max_seq, P);
-      pl->total_chunks += (P + kScoreChunk - 1) / kScoreChunk;
+      pl->total_chunks += (P + pl->chunk - 1) / pl->chunk;
     }
     pl->total_keys = p->cu_seqlens[B];
     if (need_scores) {
@@ -114,7 +115,7 @@ last_status make_plan(const last_problem *p, bool need_scores, bool need_select,
   o = align_up(o + sizeof(int32_t) * std::max(B, 1));
   const size_t blob_end = o;
   pl->off_stats = o;
-  o = align_up(o + sizeof(float) * 2 * (size_t)std::max(pl->L, 0) * std::max(pl->Hq, 0) *
+  o = align_up(o + sizeof(float) * 4 * (size_t)std::max(pl->L, 0) * std::max(pl->Hq, 0) *
                        pl->total_chunks);
   pl->off_zlog = o;
   o = align_up(o + sizeof(float) * (size_t)std::max(pl->L, 0) * std::max(pl->Hq, 0) *
@@ -123,7 +124,7 @@ last_status make_plan(const last_problem *p, bool need_scores, bool need_select,
   o = align_up(o + sizeof(float) * (size_t)pl->total_vis);
   pl->total_bytes = o;
 
-  // ---- host staging: [err words][meta][items][order], copied in one call ----
+  // ---- host staging: [err words][meta][items][order], one copy ----
   pl->blob_bytes = blob_end;
   pl->host_blob.assign(blob_end / sizeof(int32_t), 0);
   int32_t *meta = pl->host_blob.data() + pl->off_meta / 4;
@@ -141,7 +142,7 @@ last_status make_plan(const last_problem *p, bool need_scores, bool need_select,
       m[kSeqLen] = p->cu_seqlens[b + 1] - p->cu_seqlens[b];
       m[kVisStart] = p->vis_start[b];
       m[kChunkBase] = chunk;
-      const int nch = (m[kSeqLen] + kScoreChunk - 1) / kScoreChunk;
+      const int nch = (m[kSeqLen] + pl->chunk - 1) / pl->chunk;
       for (int c = 0; c < nch; ++c) {
         items[2 * (chunk + c)] = b;
         items[2 * (chunk + c) + 1] = c;

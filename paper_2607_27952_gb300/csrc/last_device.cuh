@@ -55,6 +55,13 @@ __device__ __forceinline__ U4 ldg_stream(const void *p) {
                : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w) : "l"(p));
   return r;
 }
+// Read-only load through L1 (neighbouring lanes' loads share its sectors).
+__device__ __forceinline__ U4 ldg_nc(const void *p) {
+  U4 r;
+  asm volatile("ld.global.nc.v4.u32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w) : "l"(p));
+  return r;
+}
 __device__ __forceinline__ U4 ldg(const void *p) {
   return *reinterpret_cast<const U4 *>(p);
 }

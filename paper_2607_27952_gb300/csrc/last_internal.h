@@ -24,9 +24,8 @@ enum MetaField : int {
   kMetaFields
 };
 
-constexpr int kScoreChunk = 128;     // keys per scoring CTA
 constexpr int kScoreThreads = 256;
-constexpr int kReduceThreads = 512;
+constexpr int kTokenTile = kScoreThreads;   // visual tokens per score_tokens_kernel CTA
 constexpr int kMaxGroup = 8;         // q-heads per kv-head supported by the scoring kernel
 constexpr int kMaxFeatDim = 2048;    // selection keeps x_j in 64 fp32 registers per lane
 constexpr int kSelectWarps = 8;
@@ -43,11 +42,12 @@ struct Plan {
   float scale = 0.f;
   long long total_keys = 0, total_vis = 0, total_keep = 0;
   int max_seq = 0, max_vis = 0, max_keep = 0;
+  int chunk = 0;          // keys per scoring CTA (score_chunk_keys)
   int total_chunks = 0;
   // workspace byte offsets
   size_t off_err = 0, off_meta = 0, off_items = 0, off_order = 0;
   size_t off_stats = 0, off_zlog = 0, off_w = 0, total_bytes = 0;
-  // host staging (meta rows, score items, selection order) in ws order
+  // host staging (error word, meta rows, score items, selection order) in ws order
   std::vector<int32_t> host_blob;
   size_t blob_bytes = 0;  // bytes from off_meta to the end of the order array
 };
@@ -65,6 +65,9 @@ cudaError_t launch_select(const Plan &pl, const float *w, const void *x, int32_t
                           void *x_out, char *ws, cudaStream_t s);
 cudaError_t launch_gather(const Plan &pl, const void *x, const int32_t *idx, void *x_out,
                           char *ws, cudaStream_t s);
+
+// Keys per scoring CTA for a given number of kv-heads (a multiple of 16).
+int score_chunk_keys(int num_kv_heads);
 
 // Checks the compiled limits of the scoring / selection kernels.
 bool scores_supported(const Plan &pl, std::string *why);

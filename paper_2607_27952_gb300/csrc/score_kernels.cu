@@ -1,20 +1,25 @@
 // Eq. 6-8 (Sec. 3.3): last-query-token attention scores.
 //
-// score_logits_kernel: one CTA per (request, chunk of 128 keys, layer).  It
-//   streams the chunk's keys once with 16-byte read-only loads (all kv-heads
-//   of a key are contiguous, so consecutive threads read consecutive bytes),
-//   forms the logits of the G = Hq/Hkv q-heads that share each kv-head from
-//   that single read, and writes (a) per-(layer, head, chunk) softmax
-//   statistics (max, sum of exp) and (b) the logits of the visual keys.
-//   Logits are kept in the log2 domain (q is pre-scaled by scale*log2 e).
-// score_reduce_kernel: one CTA per request.  Merges the chunk statistics of
-//   every (layer, head) in chunk order, turns each visual logit into its
-//   softmax probability, sums over layers then heads (Eq. 7), and normalises
-//   over the visual span (Eq. 8).  Fixed reduction trees: run-to-run
-//   deterministic.
+// score_logits_kernel: one CTA per (request, chunk of keys, layer), 8 warps.  A
+//   warp task is (kv-head g, 16 consecutive keys of the chunk); the two lanes of
+//   a pair share one row K[key][g][0..D): lane h of the pair reads the 16-byte
+//   segments h, h + 2, h + 4, ... so every warp-wide load fills whole 32-byte
+//   sectors, and forms partial logits of the G = Hq/Hkv q-heads of g in
+//   registers from the pre-scaled q held in shared memory (broadcast reads).
+//   One xor shuffle joins the pair.  The chunk's logits go to shared memory;
+//   per (layer, head) the CTA then writes the chunk's max and its sums of
+//   2^(z - max) over all keys and over the visual keys, and the visual logits.
+//   Logits are in the log2 domain (q pre-scaled by scale * log2 e).
+// score_tokens_kernel: one CTA per (request, 256 visual tokens).  It merges the
+//   request's chunk statistics per (layer, head) in chunk order into the max M,
+//   the total mass Z and the visual mass V, sums each visual token's
+//   probabilities over layers then heads (Eq. 7) and divides by the request's
+//   visual mass sum_lh V_lh / Z_lh (Eq. 8), which every CTA of the request
+//   computes identically.  Fixed reduction trees: run-to-run deterministic.
 #include "last_device.cuh"
 #include "last_internal.h"
 
+#include <algorithm>
 #include <cmath>
 
 namespace last {
@@ -24,251 +29,270 @@ struct ScoreArgs {
   const void *k;
   const int32_t *meta;
   const int2 *items;     // (request, chunk)
-  float2 *stats;         // [L][Hq][total_chunks]
+  float4 *stats;         // [L][Hq][total_chunks]: max, sum all, sum visual, unused
   float *zlog;           // [L][Hq][total_vis]
+  float *w;              // output scores
   long long total_keys;
   long long total_vis;
-  int L, Hq, Hkv, D, total_chunks;
+  int L, Hq, Hkv, D, total_chunks, chunk;
   float qscale;          // softmax scale * log2(e)
-  int R, log2R;          // lanes per (key, kv-head) row, power of two
-  int kpp;               // keys per pass = 256 / (Hkv * R)
 };
 
-template <typename T, int G, int SPL>
+constexpr int kSegBatch = 8;        // 16-byte loads in flight per lane
+constexpr int kRowsPerTask = 16;    // keys of one warp task (two lanes per key)
+
+template <typename T, int G>
 __global__ void __launch_bounds__(kScoreThreads)
 score_logits_kernel(const ScoreArgs a) {
-  constexpr int V = Elem<T>::kPerVec;   // elements per 16-byte vector
-  constexpr int NE = V * SPL;           // elements of one row a lane owns
-  constexpr int U = 4;                  // passes in flight per thread
-  extern __shared__ float zbuf[];       // [kScoreChunk][Hq + 1]
+  constexpr int V = Elem<T>::kPerVec;   // elements per 16-byte segment
+  extern __shared__ __align__(16) float smem_f[];
+  const int Hq = a.Hq, D = a.D;
+  float *qs = smem_f;                   // [Hq][D] pre-scaled q
+  float *zbuf = smem_f + Hq * D;        // [chunk][Hq + 1] logits
+  const int ldz = Hq + 1;
 
   const int2 item = a.items[blockIdx.x];
   const int b = item.x, chunk = item.y, l = blockIdx.y;
   const int32_t *m = a.meta + b * kMetaFields;
   const int seq0 = m[kSeqStart], P = m[kSeqLen], v0 = m[kVisStart];
   const int nvis = m[kNumVis], voff = m[kVisOff], cbase = m[kChunkBase];
-  const int p_begin = chunk * kScoreChunk;
-  const int nk = min(kScoreChunk, P - p_begin);
-  const int ldz = a.Hq + 1;
+  const int p_begin = chunk * a.chunk;
+  const int nk = min(a.chunk, P - p_begin);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
 
-  const int tid = threadIdx.x;
-  const int tpk = a.Hkv * a.R;
-  const int slot = tid / tpk;
-  const int within = tid - slot * tpk;
-  const int g = within >> a.log2R;
-  const int part = within & (a.R - 1);
-  const bool active = slot < a.kpp;
-
-  // this lane's q slice for the G heads of kv-head g, widened and pre-scaled
-  float qv[G][NE];
-  {
-    const T *qb = static_cast<const T *>(a.q) + ((long long)b * a.L + l) * a.Hq * a.D;
+  {  // q of this (request, layer), widened and pre-scaled
+    const T *qb = static_cast<const T *>(a.q) + ((long long)b * a.L + l) * Hq * D;
+    for (int v = tid; v < Hq * D / V; v += kScoreThreads) {
+      float e[V];
+      Elem<T>::widen(ldg(qb + v * V), e);
 #pragma unroll
-    for (int gg = 0; gg < G; ++gg) {
-      const T *qh = qb + (long long)(g * G + gg) * a.D;
-#pragma unroll
-      for (int j = 0; j < SPL; ++j) {
-        float e[V];
-        Elem<T>::widen(ldg(qh + (part + a.R * j) * V), e);
-#pragma unroll
-        for (int x = 0; x < V; ++x) qv[gg][j * V + x] = e[x] * a.qscale;
-      }
-    }
-  }
-
-  const T *kl = static_cast<const T *>(a.k) + ((long long)l * a.total_keys + seq0) * a.Hkv * a.D;
-  const int passes = (nk + a.kpp - 1) / a.kpp;
-  for (int pass0 = 0; pass0 < passes; pass0 += U) {
-    U4 buf[U][SPL];
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const int kk = (pass0 + u) * a.kpp + slot;
-      const bool ok = active && kk < nk;
-      const T *row = kl + ((long long)(p_begin + kk) * a.Hkv + g) * a.D;
-#pragma unroll
-      for (int j = 0; j < SPL; ++j)
-        buf[u][j] = ok ? ldg_stream(row + (part + a.R * j) * V) : U4{0, 0, 0, 0};
-    }
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      float acc[G];
-#pragma unroll
-      for (int gg = 0; gg < G; ++gg) acc[gg] = 0.f;
-#pragma unroll
-      for (int j = 0; j < SPL; ++j) {
-        float e[V];
-        Elem<T>::widen(buf[u][j], e);
-#pragma unroll
-        for (int x = 0; x < V; ++x)
-#pragma unroll
-          for (int gg = 0; gg < G; ++gg) acc[gg] = fmaf(qv[gg][j * V + x], e[x], acc[gg]);
-      }
-      for (int o = a.R >> 1; o > 0; o >>= 1)
-#pragma unroll
-        for (int gg = 0; gg < G; ++gg) acc[gg] += __shfl_xor_sync(0xffffffffu, acc[gg], o);
-      const int kk = (pass0 + u) * a.kpp + slot;
-      if (active && part == 0 && kk < nk) {
-#pragma unroll
-        for (int gg = 0; gg < G; ++gg) zbuf[kk * ldz + g * G + gg] = acc[gg];
-      }
+      for (int x = 0; x < V; ++x) qs[v * V + x] = e[x] * a.qscale;
     }
   }
   __syncthreads();
 
-  // per-head chunk statistics: max and sum of 2^(z - max)
-  const int warp = tid >> 5, lane = tid & 31;
-  for (int h = warp; h < a.Hq; h += kScoreThreads / 32) {
+  const T *kl = static_cast<const T *>(a.k) + ((long long)l * a.total_keys + seq0) * a.Hkv * D;
+  const int nseg = D / V;                 // segments per row
+  const int nhalf = (nseg + 1) >> 1;      // segments per lane of a pair
+  const int half = lane & 1, r = lane >> 1;
+  const int ngrp = (nk + kRowsPerTask - 1) / kRowsPerTask;
+  for (int task = warp; task < ngrp * a.Hkv; task += kScoreThreads / 32) {
+    const int grp = task / a.Hkv, g = task - grp * a.Hkv;
+    const int kk = grp * kRowsPerTask + r;
+    const bool ok = kk < nk;
+    const T *row = kl + ((long long)(p_begin + (ok ? kk : 0)) * a.Hkv + g) * D;
+    const float *qg = qs + g * G * D;
+    float acc[G];
+#pragma unroll
+    for (int gg = 0; gg < G; ++gg) acc[gg] = 0.f;
+    for (int s0 = 0; s0 < nhalf; s0 += kSegBatch) {
+      U4 buf[kSegBatch];
+#pragma unroll
+      for (int j = 0; j < kSegBatch; ++j) {
+        const int seg = 2 * (s0 + j) + half;
+        buf[j] = (ok && seg < nseg) ? ldg_nc(row + seg * V) : U4{0, 0, 0, 0};
+      }
+#pragma unroll
+      for (int j = 0; j < kSegBatch; ++j) {
+        const int seg = 2 * (s0 + j) + half;
+        if (seg < nseg) {
+          float e[V];
+          Elem<T>::widen(buf[j], e);
+          const float *qc = qg + seg * V;
+#pragma unroll
+          for (int gg = 0; gg < G; ++gg) {
+#pragma unroll
+            for (int x = 0; x < V; x += 4) {
+              const float4 qv = *reinterpret_cast<const float4 *>(qc + gg * D + x);
+              acc[gg] = fmaf(qv.x, e[x], acc[gg]);
+              acc[gg] = fmaf(qv.y, e[x + 1], acc[gg]);
+              acc[gg] = fmaf(qv.z, e[x + 2], acc[gg]);
+              acc[gg] = fmaf(qv.w, e[x + 3], acc[gg]);
+            }
+          }
+        }
+      }
+    }
+#pragma unroll
+    for (int gg = 0; gg < G; ++gg) acc[gg] += __shfl_xor_sync(0xffffffffu, acc[gg], 1);
+    if (ok && half == 0) {
+#pragma unroll
+      for (int gg = 0; gg < G; ++gg) zbuf[kk * ldz + g * G + gg] = acc[gg];
+    }
+  }
+  __syncthreads();
+
+  // per-head chunk statistics: max, sums of 2^(z - max) over all and over visual keys
+  const int vlo = max(p_begin, v0), vhi = min(p_begin + nk, v0 + nvis);
+  for (int h = warp; h < Hq; h += kScoreThreads / 32) {
     float mx = -INFINITY;
     for (int kk = lane; kk < nk; kk += 32) mx = fmaxf(mx, zbuf[kk * ldz + h]);
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-    float sum = 0.f;
-    for (int kk = lane; kk < nk; kk += 32) sum += exp2f(zbuf[kk * ldz + h] - mx);
+    float sum = 0.f, vis = 0.f;
+    for (int kk = lane; kk < nk; kk += 32) {
+      const float e = exp2f(zbuf[kk * ldz + h] - mx);
+      sum += e;
+      const int p = p_begin + kk;
+      if (p >= vlo && p < vhi) vis += e;
+    }
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+    for (int o = 16; o > 0; o >>= 1) {
+      sum += __shfl_xor_sync(0xffffffffu, sum, o);
+      vis += __shfl_xor_sync(0xffffffffu, vis, o);
+    }
     if (lane == 0)
-      a.stats[((long long)l * a.Hq + h) * a.total_chunks + cbase + chunk] = make_float2(mx, sum);
+      a.stats[((long long)l * Hq + h) * a.total_chunks + cbase + chunk] =
+          make_float4(mx, sum, vis, 0.f);
   }
 
   // visual logits of this chunk
-  const int vlo = max(p_begin, v0), vhi = min(p_begin + nk, v0 + nvis);
   const int nv = vhi - vlo;
   if (nv > 0) {
-    for (int idx = tid; idx < nv * a.Hq; idx += kScoreThreads) {
+    for (int idx = tid; idx < nv * Hq; idx += kScoreThreads) {
       const int h = idx / nv, i = idx - h * nv;
       const int p = vlo + i;
-      a.zlog[((long long)l * a.Hq + h) * a.total_vis + voff + (p - v0)] =
+      a.zlog[((long long)l * Hq + h) * a.total_vis + voff + (p - v0)] =
           zbuf[(p - p_begin) * ldz + h];
     }
   }
 }
 
-__global__ void __launch_bounds__(kReduceThreads)
-score_reduce_kernel(const int32_t *__restrict__ meta, const float2 *__restrict__ stats,
-                    const float *__restrict__ zlog, float *__restrict__ w, int LH,
-                    int total_chunks, long long total_vis) {
-  extern __shared__ float coef[];      // [LH] max, [LH] 1/Z
-  __shared__ float warp_sum[kReduceThreads / 32];
-  const int b = blockIdx.x;
-  const int32_t *m = meta + b * kMetaFields;
+// Eq. 7-8: one CTA per (request b, tile of kTokenTile visual tokens).
+__global__ void __launch_bounds__(kScoreThreads)
+score_tokens_kernel(const ScoreArgs a) {
+  extern __shared__ float coef[];   // [L*Hq] max, [L*Hq] 1/Z, [L*Hq] V/Z
+  __shared__ float inv_total_s;
+  const int b = blockIdx.y, tile = blockIdx.x;
+  const int32_t *m = a.meta + b * kMetaFields;
   const int nvis = m[kNumVis], voff = m[kVisOff], cbase = m[kChunkBase];
-  const int nch = (m[kSeqLen] + kScoreChunk - 1) / kScoreChunk;
-  if (nvis == 0) return;
-  float *cmax = coef, *cinv = coef + LH;
-  for (int lh = threadIdx.x; lh < LH; lh += blockDim.x) {
-    const float2 *s = stats + (long long)lh * total_chunks + cbase;
-    float mx = -INFINITY;
-    for (int c = 0; c < nch; ++c) mx = fmaxf(mx, s[c].x);
-    float z = 0.f;
-    for (int c = 0; c < nch; ++c) z += s[c].y * exp2f(s[c].x - mx);
-    cmax[lh] = mx;
-    cinv[lh] = 1.0f / z;
-  }
-  __syncthreads();
-  float local = 0.f;
-  for (int i = threadIdx.x; i < nvis; i += blockDim.x) {
-    float s = 0.f;
-    for (int lh = 0; lh < LH; ++lh)
-      s += exp2f(zlog[(long long)lh * total_vis + voff + i] - cmax[lh]) * cinv[lh];
-    w[voff + i] = s;
-    local += s;
-  }
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) local += __shfl_xor_sync(0xffffffffu, local, o);
+  if (tile * kTokenTile >= nvis) return;
+  const int nch = (m[kSeqLen] + a.chunk - 1) / a.chunk;
+  const int LH = a.L * a.Hq;
+  float *cmax = coef, *cinv = coef + LH, *cvis = coef + 2 * LH;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  if (lane == 0) warp_sum[warp] = local;
-  __syncthreads();
-  if (warp == 0) {
-    float v = lane < (int)(blockDim.x >> 5) ? warp_sum[lane] : 0.f;
+  // one warp per (layer, head): lanes stride over the request's chunks, then
+  // fixed xor trees for the max and the rescaled sums
+  for (int lh = warp; lh < LH; lh += kScoreThreads / 32) {
+    const float4 *st = a.stats + (long long)lh * a.total_chunks + cbase;
+    float mx = -INFINITY;
+    for (int c = lane; c < nch; c += 32) mx = fmaxf(mx, st[c].x);
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-    if (lane == 0) warp_sum[0] = v;
+    for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+    float z = 0.f, vz = 0.f;
+    for (int c = lane; c < nch; c += 32) {
+      const float4 v = st[c];
+      const float f = exp2f(v.x - mx);
+      z += v.y * f;
+      vz += v.z * f;
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      z += __shfl_xor_sync(0xffffffffu, z, o);
+      vz += __shfl_xor_sync(0xffffffffu, vz, o);
+    }
+    if (lane == 0) {
+      cmax[lh] = mx;
+      cinv[lh] = 1.0f / z;
+      cvis[lh] = vz / z;   // visual probability mass of (layer, head)
+    }
   }
   __syncthreads();
-  const float inv_total = 1.0f / warp_sum[0];
-  for (int i = threadIdx.x; i < nvis; i += blockDim.x) w[voff + i] = w[voff + i] * inv_total;
+  if (warp == 0) {   // sum_lh V_lh / Z_lh, strided over lanes then a fixed xor tree
+    float t = 0.f;
+    for (int lh = lane; lh < LH; lh += 32) t += cvis[lh];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+    if (lane == 0) inv_total_s = 1.0f / t;
+  }
+  __syncthreads();
+  const int i = tile * kTokenTile + threadIdx.x;
+  if (i < nvis) {
+    const float *z = a.zlog + voff + i;
+    float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+    int lh = 0;
+    for (; lh + 4 <= LH; lh += 4) {   // four independent loads in flight
+      const float z0 = z[(long long)(lh + 0) * a.total_vis];
+      const float z1 = z[(long long)(lh + 1) * a.total_vis];
+      const float z2 = z[(long long)(lh + 2) * a.total_vis];
+      const float z3 = z[(long long)(lh + 3) * a.total_vis];
+      s0 += exp2f(z0 - cmax[lh + 0]) * cinv[lh + 0];
+      s1 += exp2f(z1 - cmax[lh + 1]) * cinv[lh + 1];
+      s2 += exp2f(z2 - cmax[lh + 2]) * cinv[lh + 2];
+      s3 += exp2f(z3 - cmax[lh + 3]) * cinv[lh + 3];
+    }
+    for (; lh < LH; ++lh) s0 += exp2f(z[(long long)lh * a.total_vis] - cmax[lh]) * cinv[lh];
+    a.w[voff + i] = ((s0 + s1) + (s2 + s3)) * inv_total_s;
+  }
 }
 
 namespace {
 
-struct ScoreShape {
-  int spl, R, log2R, kpp;
-};
-
-bool score_shape(const Plan &pl, ScoreShape *sh, std::string *why) {
-  const int V = 16 / pl.elem;
-  if (pl.D % V) { if (why) *why = "head_dim * elem_bytes must be a multiple of 16"; return false; }
-  const int segs = pl.D / V;            // 16-byte vectors per (key, kv-head) row
-  if (segs & (segs - 1)) {
-    if (why) *why = "head_dim * elem_bytes must be 16 bytes times a power of two";
-    return false;
-  }
-  int spl = pl.G <= 2 ? 2 : 1;
-  if (spl > segs) spl = segs;
-  const int R = segs / spl;
-  if (R > 32) { if (why) *why = "head_dim * elem_bytes must be <= 512 (G>2) or 1024 bytes"; return false; }
-  if (pl.Hkv * R > kScoreThreads) {
-    if (why) *why = "num_kv_heads * head_dim * elem_bytes too large for one scoring CTA";
-    return false;
-  }
-  int log2R = 0;
-  while ((1 << log2R) < R) ++log2R;
-  *sh = ScoreShape{spl, R, log2R, kScoreThreads / (pl.Hkv * R)};
-  return true;
-}
-
-template <typename T, int G>
-void *pick_logits(int spl) {
-  return spl == 2 ? (void *)score_logits_kernel<T, G, 2> : (void *)score_logits_kernel<T, G, 1>;
-}
-
 template <typename T>
-void *pick_logits_g(int G, int spl) {
+void *pick_logits(int G) {
   switch (G) {
-    case 1: return pick_logits<T, 1>(spl);
-    case 2: return pick_logits<T, 2>(spl);
-    case 3: return (void *)score_logits_kernel<T, 3, 1>;
-    case 4: return (void *)score_logits_kernel<T, 4, 1>;
-    case 5: return (void *)score_logits_kernel<T, 5, 1>;
-    case 6: return (void *)score_logits_kernel<T, 6, 1>;
-    case 7: return (void *)score_logits_kernel<T, 7, 1>;
-    case 8: return (void *)score_logits_kernel<T, 8, 1>;
+    case 1: return (void *)score_logits_kernel<T, 1>;
+    case 2: return (void *)score_logits_kernel<T, 2>;
+    case 3: return (void *)score_logits_kernel<T, 3>;
+    case 4: return (void *)score_logits_kernel<T, 4>;
+    case 5: return (void *)score_logits_kernel<T, 5>;
+    case 6: return (void *)score_logits_kernel<T, 6>;
+    case 7: return (void *)score_logits_kernel<T, 7>;
+    case 8: return (void *)score_logits_kernel<T, 8>;
   }
   return nullptr;
 }
 
+size_t logits_smem(const Plan &pl) {
+  return sizeof(float) * ((size_t)pl.Hq * pl.D + (size_t)pl.chunk * (pl.Hq + 1));
+}
+
+constexpr size_t kMaxScoreSmem = 100 * 1024;
+
 }  // namespace
+
+int score_chunk_keys(int num_kv_heads) {
+  // about 32 (kv-head, 16-key) warp tasks per CTA, 16..256 keys
+  int c = 512 / std::max(num_kv_heads, 1) / kRowsPerTask * kRowsPerTask;
+  return std::min(256, std::max(kRowsPerTask, c));
+}
 
 bool scores_supported(const Plan &pl, std::string *why) {
   if (pl.G < 1 || pl.G > kMaxGroup) {
     if (why) *why = "num_q_heads / num_kv_heads must be in [1, 8]";
     return false;
   }
-  ScoreShape sh;
-  return score_shape(pl, &sh, why);
+  if ((pl.D * pl.elem) % 16) {
+    if (why) *why = "head_dim * elem_bytes must be a multiple of 16";
+    return false;
+  }
+  if (logits_smem(pl) > kMaxScoreSmem) {
+    if (why) *why = "num_q_heads * head_dim too large for the scoring kernel's shared memory";
+    return false;
+  }
+  return true;
 }
 
 cudaError_t launch_scores(const Plan &pl, const void *q, const void *k, float *w_out, char *ws,
                           cudaStream_t s) {
   if (pl.total_vis == 0 || pl.B == 0) return cudaSuccess;
-  ScoreShape sh;
-  score_shape(pl, &sh, nullptr);
   ScoreArgs a;
   a.q = q;
   a.k = k;
   a.meta = reinterpret_cast<const int32_t *>(ws + pl.off_meta);
   a.items = reinterpret_cast<const int2 *>(ws + pl.off_items);
-  a.stats = reinterpret_cast<float2 *>(ws + pl.off_stats);
+  a.stats = reinterpret_cast<float4 *>(ws + pl.off_stats);
   a.zlog = reinterpret_cast<float *>(ws + pl.off_zlog);
+  a.w = w_out;
   a.total_keys = pl.total_keys;
   a.total_vis = pl.total_vis;
   a.L = pl.L; a.Hq = pl.Hq; a.Hkv = pl.Hkv; a.D = pl.D;
   a.total_chunks = pl.total_chunks;
+  a.chunk = pl.chunk;
   a.qscale = pl.scale * 1.4426950408889634f;
-  a.R = sh.R; a.log2R = sh.log2R; a.kpp = sh.kpp;
-  void *fn = pl.dtype == LAST_DTYPE_BF16 ? pick_logits_g<__nv_bfloat16>(pl.G, sh.spl)
-                                         : pick_logits_g<float>(pl.G, sh.spl);
-  const size_t smem = sizeof(float) * kScoreChunk * (pl.Hq + 1);
+  void *fn = pl.dtype == LAST_DTYPE_BF16 ? pick_logits<__nv_bfloat16>(pl.G)
+                                         : pick_logits<float>(pl.G);
+  const size_t smem = logits_smem(pl);
   cudaError_t e;
   if (smem > 48 * 1024) {
     e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
@@ -277,9 +301,14 @@ cudaError_t launch_scores(const Plan &pl, const void *q, const void *k, float *w
   void *args[] = {&a};
   e = cudaLaunchKernel(fn, dim3(pl.total_chunks, pl.L), dim3(kScoreThreads), args, smem, s);
   if (e != cudaSuccess) return e;
-  const int LH = pl.L * pl.Hq;
-  score_reduce_kernel<<<pl.B, kReduceThreads, sizeof(float) * 2 * LH, s>>>(
-      a.meta, a.stats, a.zlog, w_out, LH, pl.total_chunks, pl.total_vis);
+  const int max_tiles = (pl.max_vis + kTokenTile - 1) / kTokenTile;
+  const size_t tsmem = sizeof(float) * 3 * pl.L * pl.Hq;
+  if (tsmem > 48 * 1024) {
+    e = cudaFuncSetAttribute(score_tokens_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)tsmem);
+    if (e != cudaSuccess) return e;
+  }
+  score_tokens_kernel<<<dim3(max_tiles, pl.B), kScoreThreads, tsmem, s>>>(a);
   return cudaGetLastError();
 }
 

@@ -58,7 +58,9 @@ def test_workspace_size_is_host_only(lib):
     (dict(cu_seqlens=[0, 0, 30], vis_start=[0, 2], cu_vis=[0, 0, 14],
           cu_keep=[0, 0, 5]), last.LAST_ERR_INVALID_ARG),                    # P_b = 0
     (dict(num_q_heads=18, num_kv_heads=2), last.LAST_ERR_UNSUPPORTED),       # G = 9 > 8
-    (dict(head_dim=80), last.LAST_ERR_UNSUPPORTED),                          # 160 B rows
+    (dict(head_dim=12), last.LAST_ERR_UNSUPPORTED),                          # 24 B rows
+    (dict(num_q_heads=256, num_kv_heads=32, head_dim=128),
+     last.LAST_ERR_UNSUPPORTED),                                             # q > smem
 ])
 def test_scores_rejects_bad_problems_before_launch(lib, kw, status):
     prob = _problem(**kw)
