@@ -77,6 +77,8 @@ def _load():
         lib.oracle_select_fp32.restype = i32
         lib.oracle_select_fp64.argtypes = [i32, i32, i32, P, P, i32, P]
         lib.oracle_select_fp64.restype = i32
+        lib.oracle_select_topk.argtypes = [i32, P, i32, P]
+        lib.oracle_select_topk.restype = i32
         lib.oracle_restore_order.argtypes = [i32, P, P]
         lib.oracle_restore_order.restype = None
         lib.oracle_gather.argtypes = [i32, i32, i32, P, i32, P, P]
@@ -156,6 +158,17 @@ def select_fp64(x, w, k):
     rc = _load().oracle_select_fp64(N, d, _dtype_code(x), _ptr(x), _ptr(w), int(k), _ptr(out))
     if rc:
         raise ValueError(f"oracle_select_fp64 rejected its arguments (rc={rc})")
+    return out[:k]
+
+
+def select_topk(w, k):
+    """Table 5's Top-k selection: the k highest scores, ties to the lowest index.
+    Returns the selection order (descending score, int32)."""
+    w = np.ascontiguousarray(np.asarray(w, dtype=np.float32))
+    out = np.zeros(max(k, 1), dtype=np.int32)
+    rc = _load().oracle_select_topk(len(w), _ptr(w), int(k), _ptr(out))
+    if rc:
+        raise ValueError(f"oracle_select_topk rejected its arguments (rc={rc})")
     return out[:k]
 
 

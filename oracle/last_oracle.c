@@ -14,6 +14,7 @@
  *   oracle_scores          Eq. 6, 7, 8 (sum over layers and heads, normalise)
  *   oracle_select_fp32     Eq. 9, 10, 11 in "canonical fp32" arithmetic
  *   oracle_select_fp64     Eq. 9, 10, 11 in plain fp64 arithmetic
+ *   oracle_select_topk     Table 5's "Top-k" selection: the k highest scores
  *   oracle_restore_order   Eq. 12 (sort(S))
  *   oracle_gather          Eq. 12 (X_S = [x_i], i in sort(S))
  *   oracle_budget          Eq. 2  (K = ceil(rho N))
@@ -272,6 +273,28 @@ int oracle_select_fp64(int N, int d, int dtype, const void *x, const double *w, 
     in_s[j] = 1;
   }
   free(xd); free(r); free(delta); free(in_s);
+  return 0;
+}
+
+/* Table 5 ("LAST (Top-k)"): keep the k tokens with the highest importance
+ * score w~, with no diversity term.  Written as k repeated argmaxes over the
+ * tokens not yet taken (ties to the lowest index, IEEE '>' so -0 == +0), which
+ * is the greedy of Eq. 9-11 with every delta fixed at 1.  order_out receives
+ * the selection order (descending score). */
+int oracle_select_topk(int N, const float *w, int k, int32_t *order_out) {
+  if (N < 0 || k < 0 || k > N) return 1;
+  unsigned char *taken = (unsigned char *)calloc((size_t)N + 1, 1);
+  if (!taken) return 2;
+  for (int t = 0; t < k; ++t) {
+    int best = -1;
+    for (int i = 0; i < N; ++i) {
+      if (taken[i]) continue;
+      if (best < 0 || w[i] > w[best]) best = i;
+    }
+    order_out[t] = best;
+    taken[best] = 1;
+  }
+  free(taken);
   return 0;
 }
 

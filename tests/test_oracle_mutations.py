@@ -33,10 +33,15 @@ MUTANTS = [
      "  int j = 0;\n  order_out[0] = j;\n  in_s[j] = 1;\n  for (int t = 1; t < k; ++t) {\n    /* Eq. 10"),
     ("order_not_restored", "while (b >= 0 && idx_out[b] > v)", "while (b >= 0 && idx_out[b] < v)"),
     ("budget_floor", "if (q * den < prod) q += 1;", ""),
+    ("topk_tie_to_highest_index", "if (best < 0 || w[i] > w[best]) best = i;",
+     "if (best < 0 || w[i] >= w[best]) best = i;"),
+    ("topk_lowest_scores", "if (best < 0 || w[i] > w[best]) best = i;",
+     "if (best < 0 || w[i] < w[best]) best = i;"),
 ]
 
 PIN_FILES = [os.path.join(ROOT, "tests", "test_oracle_scores.py"),
-             os.path.join(ROOT, "tests", "test_oracle_select.py")]
+             os.path.join(ROOT, "tests", "test_oracle_select.py"),
+             os.path.join(ROOT, "tests", "test_oracle_topk.py")]
 
 
 def _run_pins(lib):
