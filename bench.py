@@ -47,6 +47,9 @@ def parse():
     ap.add_argument("--budget", default="mixed", help="c2 budget: mixed, 64, 128 or 192")
     ap.add_argument("--workload", default="c2", choices=["c1", "c2", "c3", "c4", "c5"],
                     help="c2 (default) is the benchmark line; the others are reported for context")
+    ap.add_argument("--selector", default="greedy", choices=["greedy", "topk"],
+                    help="greedy: importance-weighted k-center (Eq. 9-11, the method); "
+                         "topk: the Top-k variant of Table 5")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     return ap.parse_args()
@@ -233,28 +236,37 @@ def peaks():
         return {"hbm_gbs": FALLBACK_HBM_GBS, "sm_max_mhz": 2070.0}, "fallback"
 
 
-def cpu_baseline(wl, budget_s=15.0):
+def oracle_request(oracle, wl, b, selector="greedy"):
+    """One whole request through the oracle: fp64 scores of the request, then the
+    canonical-fp32 greedy (or Top-k), order restore and gather.  Returns N_b."""
+    v0, v1 = int(wl.cu_vis[b]), int(wl.cu_vis[b + 1])
+    s0, s1 = int(wl.cu_seqlens[b]), int(wl.cu_seqlens[b + 1])
+    kb = int(wl.cu_keep[b + 1] - wl.cu_keep[b])
+    w = oracle.scores(wl.q[b:b + 1], np.ascontiguousarray(wl.k[:, s0:s1]), [0, s1 - s0],
+                      [int(wl.vis_start[b])], [0, v1 - v0], num_kv_heads=wl.num_kv_heads)
+    w32 = w.astype(np.float32)
+    if selector == "topk":
+        oracle.gather(wl.x[v0:v1], oracle.restore_order(oracle.select_topk(w32, kb)))
+    else:
+        oracle.prune_request(wl.x[v0:v1], w32, kb)
+    return v1 - v0
+
+
+def cpu_baseline(wl, budget_s=15.0, selector="greedy"):
     """The oracle as it stands (single thread) on a bounded sample of the same batch:
-    whole requests (fp64 scores of the request, canonical-fp32 greedy, gather)."""
+    whole requests in batch order until about budget_s seconds have passed."""
     import oracle
-    from workloads import custom  # noqa: F401  (same generator as the GPU leg)
     oracle.build()
     t0 = time.perf_counter()
     done = 0
-    order = [0, 1, 2] * (wl.batch // 3)
-    for b in order:
-        v0, v1 = int(wl.cu_vis[b]), int(wl.cu_vis[b + 1])
-        s0, s1 = int(wl.cu_seqlens[b]), int(wl.cu_seqlens[b + 1])
-        kb = int(wl.cu_keep[b + 1] - wl.cu_keep[b])
-        w = oracle.scores(wl.q[b:b + 1], np.ascontiguousarray(wl.k[:, s0:s1]), [0, s1 - s0],
-                          [int(wl.vis_start[b])], [0, v1 - v0], num_kv_heads=wl.num_kv_heads)
-        oracle.prune_request(wl.x[v0:v1], w.astype(np.float32), kb)
+    for b in range(wl.batch):
+        oracle_request(oracle, wl, b, selector)
         done += 1
         if time.perf_counter() - t0 > budget_s:
             break
     dt = time.perf_counter() - t0
     return {"value": done / dt, "unit": UNIT, "cores": 1, "kind": "oracle",
-            "sample": f"{done} whole requests of the same batch (k=64/128/192 in turn), "
+            "sample": f"the first {done} whole requests of the same batch ({selector}), "
                       f"single-threaded C oracle, {dt:.1f} s"}
 
 
@@ -262,20 +274,13 @@ def run_reference(args, rank, world):
     """--impl reference: the oracle, as it stands, on the host cores (rank 0 only)."""
     if rank != 0:
         return
-    wl = workload(args.budget, 0)
+    wl = workload(args.budget, 0, args.workload)
     import oracle
     oracle.build()
 
     def step(i):
-        # a bounded sample per step: one whole request, budgets in turn
-        b = i % 3
-        v0, v1 = int(wl.cu_vis[b]), int(wl.cu_vis[b + 1])
-        s0, s1 = int(wl.cu_seqlens[b]), int(wl.cu_seqlens[b + 1])
-        kb = int(wl.cu_keep[b + 1] - wl.cu_keep[b])
-        w = oracle.scores(wl.q[b:b + 1], np.ascontiguousarray(wl.k[:, s0:s1]), [0, s1 - s0],
-                          [int(wl.vis_start[b])], [0, v1 - v0], num_kv_heads=wl.num_kv_heads)
-        oracle.prune_request(wl.x[v0:v1], w.astype(np.float32), kb)
-        return v1 - v0
+        # a bounded sample per step: one whole request of the batch, in turn
+        return oracle_request(oracle, wl, i % wl.batch, args.selector)
 
     for i in range(args.warmup):
         step(i)
@@ -289,10 +294,12 @@ def run_reference(args, rank, world):
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": 1000 * dt / args.steps, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64 scores / f32 selection", "data": "synthetic",
-            "config": workload_desc(wl, args.budget) | {"per_step": "1 whole request (oracle)"},
+            "config": workload_desc(wl, args.budget, args.workload)
+                      | {"per_step": "1 whole request (oracle)", "selector": args.selector},
             "visual_tokens_scored_per_s": toks / dt,
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
-                             "sample": "1 whole request of the c2 batch per step, budgets in turn"},
+                             "sample": f"1 whole request of the {args.workload} batch per step, "
+                                       "requests in turn"},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
@@ -336,9 +343,17 @@ def main():
     ws = last.workspace(prob, dev)
     stream = torch.cuda.current_stream(dev)
 
+    topk = args.selector == "topk"
+
+    def select():
+        if topk:
+            last.last_select_topk(prob, w, idx, ws, stream, x=x, x_out=xs)
+        else:
+            last.last_select(prob, w, x, idx, ws, stream, x_out=xs)
+
     def step():
         last.last_scores(prob, q, k, w, ws, stream)
-        last.last_select(prob, w, x, idx, ws, stream, x_out=xs)
+        select()
 
     for _ in range(args.warmup):
         step()
@@ -357,7 +372,7 @@ def main():
             ev[i][0].record(stream)
             last.last_scores(prob, q, k, w, ws, stream)
             ev[i][1].record(stream)
-            last.last_select(prob, w, x, idx, ws, stream, x_out=xs)
+            select()
             ev[i][2].record(stream)
         torch.cuda.synchronize(dev)
         barrier()
@@ -384,6 +399,8 @@ def main():
         e2e = measure_e2e(args, wl, prob, dev, stream, last, q, k, x)
 
     comp, greedy = prune_bytes_moved(wl)
+    if topk:   # Top-k reads only the kept rows of X, and has no greedy reads
+        comp, greedy = comp - wl.x.nbytes, 0
     moved_tbs = (comp + greedy) / (total_ms / K / 1e3) / 1e12
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
@@ -392,12 +409,13 @@ def main():
         "data": "synthetic (seeded; shapes of the paper's LLaVA-1.5 workload)",
         "config": workload_desc(wl, args.budget, args.workload) | {"parallelism": f"replicas x{world}"},
         "visual_tokens_scored_per_s": tokens_per_s,
-        "gpu_launches": 3 * K,
+        "gpu_launches": (4 if topk else 3) * K,
         "kernels": {"scores_ms": scores_ms, "select_ms": select_ms,
                     "scores_GBps": sc_gbs, "scores_hbm_frac": sc_gbs / hbm},
         "roofline": {"bound": "alu", "kernel": "select_kernel", "achieved": achieved,
                      "peak": alu_peak_tflops, "unit": "TFLOP/s", "frac": achieved / alu_peak_tflops,
-                     "traffic": measured_traffic("select_kernels.cu", f"c2-{args.budget}"),
+                     "traffic": measured_traffic("select_kernels.cu",
+                                                 f"{args.workload}-{args.budget}"),
                      "peak_note": f"{sm_count} SMs x {FP32_LANES_PER_SM} fp32 FMA/clk x 2 x "
                                   f"{sm_max:.0f} MHz ({pk_kind} max clock)"},
         "clocks": clocks,
@@ -407,10 +425,19 @@ def main():
                               "note": "bytes-moved accounting of the 70% HBM target; the greedy "
                                       "reads are served from shared memory / L2"},
     }
+    if topk:
+        # the selection is a few microseconds; the scoring pair dominates the step
+        line["config"]["selector"] = "topk (Table 5)"
+        line["roofline"] = {"bound": "hbm", "kernel": "score_logits_kernel+score_tokens_kernel",
+                            "achieved": sc_gbs, "peak": hbm, "unit": "GB/s", "frac": sc_gbs / hbm,
+                            "traffic": None,
+                            "peak_note": f"{pk_kind} HBM copy bandwidth; achieved = compulsory "
+                                         "scoring bytes / event time of last_scores"}
+        line["kernels"]["topk_gather_ms"] = line["kernels"].pop("select_ms")
     if e2e is not None:
         line["e2e"] = e2e
     if rank == 0 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(wl)
+        line["cpu_baseline"] = cpu_baseline(wl, selector=args.selector)
     if rank == 0:
         print(json.dumps(line), flush=True)
     if world > 1:
@@ -434,11 +461,17 @@ def measure_e2e(args, wl, prob, dev, stream, last, q_d, k_d, x_d):
     xs_d = torch.empty((nkeep, wl.feat_dim), dtype=xh.dtype, device=dev)
     ws = last.workspace(prob, dev)
 
+    w_d = torch.empty(int(wl.cu_vis[-1]), dtype=torch.float32, device=dev)
+
     def step():
         q_d.copy_(qh, non_blocking=True)
         k_d.copy_(kh, non_blocking=True)
         x_d.copy_(xh, non_blocking=True)
-        last.last_prune(prob, q_d, k_d, x_d, None, idx_d, xs_d, ws, stream)
+        if args.selector == "topk":
+            last.last_scores(prob, q_d, k_d, w_d, ws, stream)
+            last.last_select_topk(prob, w_d, idx_d, ws, stream, x=x_d, x_out=xs_d)
+        else:
+            last.last_prune(prob, q_d, k_d, x_d, None, idx_d, xs_d, ws, stream)
         idx_h.copy_(idx_d, non_blocking=True)
         xs_h.copy_(xs_d, non_blocking=True)
 

@@ -112,6 +112,18 @@ last_status last_select(const last_problem *p, const float *w, const void *x,
                         int32_t *idx_out, void *x_out, void *ws, size_t ws_bytes,
                         void *stream);
 
+/* Table 5, "LAST (Top-k)": the selection variant without the diversity term.
+ * idx_out [cu_keep[batch]] receives, per request and in ascending order, the
+ * k_b indices of highest w~ (ties between equal scores go to the lower index;
+ * -0 equals +0).  When x_out is not NULL the kept rows of x are also written
+ * there (x is then required; feat_dim a positive multiple of 8); x may be NULL
+ * otherwise.  The problem's layer/head fields are not used.  Same ownership,
+ * stream and error rules as last_select.  w must hold no NaN: the kept set is
+ * then unspecified (but still k_b distinct valid indices). */
+last_status last_select_topk(const last_problem *p, const float *w, const void *x,
+                             int32_t *idx_out, void *x_out, void *ws, size_t ws_bytes,
+                             void *stream);
+
 /* Eq. 12.  x_out[r] = x[cu_vis[b] + idx[r]] for r in request b's output range.
  * An index outside [0, N_b) leaves its row unwritten and makes last_poll
  * return LAST_ERR_DEVICE_INDEX. */

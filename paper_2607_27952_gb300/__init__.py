@@ -6,8 +6,9 @@ C problem struct.  There is no CPU fallback: if the library is missing, every
 call raises.
 
 Functions carry the names of the C entry points in include/last.h:
-  last_workspace_size, last_scores, last_select, last_gather, last_prune,
-  last_poll, last_budget, last_status_string.
+  last_workspace_size, last_scores, last_select, last_select_topk, last_gather,
+  last_prune, last_scores_noalloc, last_poll, last_budget, last_status_string,
+  last_error_message.
 """
 from __future__ import annotations
 
@@ -33,7 +34,7 @@ LAST_DTYPE_BF16 = 1
 
 EXPORTED = ("last_workspace_size", "last_scores", "last_select", "last_gather", "last_prune",
             "last_poll", "last_budget", "last_status_string", "last_error_message",
-            "last_scores_noalloc")
+            "last_scores_noalloc", "last_select_topk")
 
 
 class LastError(RuntimeError):
@@ -75,6 +76,7 @@ def load_library(path: str = LIB_PATH):
     lib.last_scores.argtypes = [PP, P, P, P, P, ctypes.c_size_t, P]
     lib.last_select.argtypes = [PP, P, P, P, P, P, ctypes.c_size_t, P]
     lib.last_gather.argtypes = [PP, P, P, P, P, ctypes.c_size_t, P]
+    lib.last_select_topk.argtypes = [PP, P, P, P, P, P, ctypes.c_size_t, P]
     lib.last_prune.argtypes = [PP, P, P, P, P, P, P, P, ctypes.c_size_t, P]
     lib.last_poll.argtypes = [P, P]
     lib.last_scores_noalloc.argtypes = [PP, P, P, P, P]
@@ -85,7 +87,7 @@ def load_library(path: str = LIB_PATH):
     lib.last_error_message.argtypes = []
     lib.last_error_message.restype = ctypes.c_char_p
     for name in ("last_workspace_size", "last_scores", "last_select", "last_gather",
-                 "last_prune", "last_poll", "last_scores_noalloc"):
+                 "last_prune", "last_poll", "last_scores_noalloc", "last_select_topk"):
         getattr(lib, name).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -188,6 +190,12 @@ def last_select(problem: Problem, w, x, idx_out, ws, stream=None, x_out=None):
     p, n = _ws(ws)
     _check(load_library().last_select(problem.ref, _ptr(w), _ptr(x), _ptr(idx_out), _ptr(x_out),
                                       p, n, _stream(stream)))
+
+
+def last_select_topk(problem: Problem, w, idx_out, ws, stream=None, x=None, x_out=None):
+    p, n = _ws(ws)
+    _check(load_library().last_select_topk(problem.ref, _ptr(w), _ptr(x), _ptr(idx_out),
+                                           _ptr(x_out), p, n, _stream(stream)))
 
 
 def last_gather(problem: Problem, x, idx, x_out, ws, stream=None):

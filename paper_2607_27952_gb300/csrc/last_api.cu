@@ -235,6 +235,35 @@ last_status last_select(const last_problem *p, const float *w, const void *x, in
   return LAST_OK;
 }
 
+last_status last_select_topk(const last_problem *p, const float *w, const void *x,
+                             int32_t *idx_out, void *x_out, void *ws, size_t ws_bytes,
+                             void *stream) {
+  Plan pl;
+  last_status st = make_plan(p, false, false, &pl);
+  if (st != LAST_OK) return st;
+  if ((st = check_ws(pl, ws, ws_bytes)) != LAST_OK) return st;
+  if (pl.total_keep > 0 && (w == nullptr || idx_out == nullptr))
+    return fail(LAST_ERR_INVALID_ARG, "w and idx_out are required");
+  if (x_out != nullptr) {
+    if (p->feat_dim < 8 || p->feat_dim % 8 != 0)
+      return fail(LAST_ERR_INVALID_ARG, "feat_dim must be a positive multiple of 8");
+    if (pl.total_keep > 0 && x == nullptr)
+      return fail(LAST_ERR_INVALID_ARG, "x is required when x_out is given");
+    if (!aligned16(x) || !aligned16(x_out))
+      return fail(LAST_ERR_INVALID_ARG, "x and x_out must be 16-byte aligned");
+  }
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if ((st = stage(pl, ws, s)) != LAST_OK) return st;
+  char *wsc = static_cast<char *>(ws);
+  cudaError_t e = launch_topk(pl, w, idx_out, wsc, s);
+  if (e != cudaSuccess) return cuda_fail(e, "top-k launch");
+  if (x_out != nullptr) {
+    e = launch_gather(pl, x, idx_out, x_out, wsc, s);
+    if (e != cudaSuccess) return cuda_fail(e, "gather launch");
+  }
+  return LAST_OK;
+}
+
 last_status last_gather(const last_problem *p, const void *x, const int32_t *idx, void *x_out,
                         void *ws, size_t ws_bytes, void *stream) {
   Plan pl;

@@ -65,6 +65,8 @@ cudaError_t launch_select(const Plan &pl, const float *w, const void *x, int32_t
                           void *x_out, char *ws, cudaStream_t s);
 cudaError_t launch_gather(const Plan &pl, const void *x, const int32_t *idx, void *x_out,
                           char *ws, cudaStream_t s);
+cudaError_t launch_topk(const Plan &pl, const float *w, int32_t *idx_out, char *ws,
+                        cudaStream_t s);
 
 // Keys per scoring CTA for a given number of kv-heads (a multiple of 16).
 int score_chunk_keys(int num_kv_heads);

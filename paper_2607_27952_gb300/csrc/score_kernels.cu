@@ -21,6 +21,9 @@
 
 #include <algorithm>
 #include <cmath>
+#include <map>
+#include <mutex>
+#include <tuple>
 
 namespace last {
 
@@ -42,7 +45,7 @@ constexpr int kSegBatch = 8;        // 16-byte loads in flight per lane
 constexpr int kRowsPerTask = 16;    // keys of one warp task (two lanes per key)
 
 template <typename T, int G>
-__global__ void __launch_bounds__(kScoreThreads)
+__global__ void __launch_bounds__(kScoreThreads, 3)
 score_logits_kernel(const ScoreArgs a) {
   constexpr int V = Elem<T>::kPerVec;   // elements per 16-byte segment
   extern __shared__ __align__(16) float smem_f[];
@@ -50,112 +53,139 @@ score_logits_kernel(const ScoreArgs a) {
   float *qs = smem_f;                   // [Hq][D] pre-scaled q
   float *zbuf = smem_f + Hq * D;        // [chunk][Hq + 1] logits
   const int ldz = Hq + 1;
-
-  const int2 item = a.items[blockIdx.x];
-  const int b = item.x, chunk = item.y, l = blockIdx.y;
-  const int32_t *m = a.meta + b * kMetaFields;
-  const int seq0 = m[kSeqStart], P = m[kSeqLen], v0 = m[kVisStart];
-  const int nvis = m[kNumVis], voff = m[kVisOff], cbase = m[kChunkBase];
-  const int p_begin = chunk * a.chunk;
-  const int nk = min(a.chunk, P - p_begin);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-
-  {  // q of this (request, layer), widened and pre-scaled
-    const T *qb = static_cast<const T *>(a.q) + ((long long)b * a.L + l) * Hq * D;
-    for (int v = tid; v < Hq * D / V; v += kScoreThreads) {
-      float e[V];
-      Elem<T>::widen(ldg(qb + v * V), e);
-#pragma unroll
-      for (int x = 0; x < V; ++x) qs[v * V + x] = e[x] * a.qscale;
-    }
-  }
-  __syncthreads();
-
-  const T *kl = static_cast<const T *>(a.k) + ((long long)l * a.total_keys + seq0) * a.Hkv * D;
   const int nseg = D / V;                 // segments per row
   const int nhalf = (nseg + 1) >> 1;      // segments per lane of a pair
   const int half = lane & 1, r = lane >> 1;
-  const int ngrp = (nk + kRowsPerTask - 1) / kRowsPerTask;
-  for (int task = warp; task < ngrp * a.Hkv; task += kScoreThreads / 32) {
-    const int grp = task / a.Hkv, g = task - grp * a.Hkv;
-    const int kk = grp * kRowsPerTask + r;
-    const bool ok = kk < nk;
-    const T *row = kl + ((long long)(p_begin + (ok ? kk : 0)) * a.Hkv + g) * D;
-    const float *qg = qs + g * G * D;
-    float acc[G];
-#pragma unroll
-    for (int gg = 0; gg < G; ++gg) acc[gg] = 0.f;
-    for (int s0 = 0; s0 < nhalf; s0 += kSegBatch) {
-      U4 buf[kSegBatch];
+  const int total_items = a.total_chunks * a.L;
+
+  // persistent: items (layer-major, then request chunks) strided over the grid
+  for (int it = blockIdx.x; it < total_items; it += gridDim.x) {
+    const int l = it / a.total_chunks;
+    const int2 item = a.items[it - l * a.total_chunks];
+    const int b = item.x, chunk = item.y;
+    const int32_t *m = a.meta + b * kMetaFields;
+    const int seq0 = m[kSeqStart], P = m[kSeqLen], v0 = m[kVisStart];
+    const int nvis = m[kNumVis], voff = m[kVisOff], cbase = m[kChunkBase];
+    const int p_begin = chunk * a.chunk;
+    const int nk = min(a.chunk, P - p_begin);
+    const int ngrp = (nk + kRowsPerTask - 1) / kRowsPerTask;
+    const int ntask = ngrp * a.Hkv;
+    const T *kl = static_cast<const T *>(a.k) + ((long long)l * a.total_keys + seq0) * a.Hkv * D;
+
+    auto row_of = [&](int task, bool *ok, int *kk, int *g) {
+      const int grp = task / a.Hkv;
+      *g = task - grp * a.Hkv;
+      *kk = grp * kRowsPerTask + r;
+      *ok = *kk < nk;
+      return kl + ((long long)(p_begin + (*ok ? *kk : 0)) * a.Hkv + *g) * D;
+    };
+    auto issue = [&](const T *row, bool ok, int s0, U4 *buf) {
 #pragma unroll
       for (int j = 0; j < kSegBatch; ++j) {
         const int seg = 2 * (s0 + j) + half;
         buf[j] = (ok && seg < nseg) ? ldg_nc(row + seg * V) : U4{0, 0, 0, 0};
       }
+    };
+
+    // the first key batch is in flight while q is staged
+    U4 buf[kSegBatch];
+    {
+      bool ok = false;
+      int kk, g;
+      const T *row = warp < ntask ? row_of(warp, &ok, &kk, &g) : kl;
+      issue(row, ok && warp < ntask, 0, buf);
+    }
+    __syncthreads();   // the previous item is done with qs and zbuf
+    {
+      const T *qb = static_cast<const T *>(a.q) + ((long long)b * a.L + l) * Hq * D;
+      for (int v = tid; v < Hq * D / V; v += kScoreThreads) {
+        float e[V];
+        Elem<T>::widen(ldg(qb + v * V), e);
 #pragma unroll
-      for (int j = 0; j < kSegBatch; ++j) {
-        const int seg = 2 * (s0 + j) + half;
-        if (seg < nseg) {
-          float e[V];
-          Elem<T>::widen(buf[j], e);
-          const float *qc = qg + seg * V;
+        for (int x = 0; x < V; ++x) qs[v * V + x] = e[x] * a.qscale;
+      }
+    }
+    __syncthreads();
+
+    for (int task = warp; task < ntask; task += kScoreThreads / 32) {
+      bool ok;
+      int kk, g;
+      const T *row = row_of(task, &ok, &kk, &g);
+      const float *qg = qs + g * G * D;
+      float acc[G];
 #pragma unroll
-          for (int gg = 0; gg < G; ++gg) {
+      for (int gg = 0; gg < G; ++gg) acc[gg] = 0.f;
+      for (int s0 = 0; s0 < nhalf; s0 += kSegBatch) {
+        if (task != warp || s0 != 0) issue(row, ok, s0, buf);
 #pragma unroll
-            for (int x = 0; x < V; x += 4) {
-              const float4 qv = *reinterpret_cast<const float4 *>(qc + gg * D + x);
-              acc[gg] = fmaf(qv.x, e[x], acc[gg]);
-              acc[gg] = fmaf(qv.y, e[x + 1], acc[gg]);
-              acc[gg] = fmaf(qv.z, e[x + 2], acc[gg]);
-              acc[gg] = fmaf(qv.w, e[x + 3], acc[gg]);
+        for (int j = 0; j < kSegBatch; ++j) {
+          const int seg = 2 * (s0 + j) + half;
+          if (seg < nseg) {
+            float e[V];
+            Elem<T>::widen(buf[j], e);
+            const float *qc = qg + seg * V;
+#pragma unroll
+            for (int gg = 0; gg < G; ++gg) {
+#pragma unroll
+              for (int x = 0; x < V; x += 4) {
+                const float4 qv = *reinterpret_cast<const float4 *>(qc + gg * D + x);
+                acc[gg] = fmaf(qv.x, e[x], acc[gg]);
+                acc[gg] = fmaf(qv.y, e[x + 1], acc[gg]);
+                acc[gg] = fmaf(qv.z, e[x + 2], acc[gg]);
+                acc[gg] = fmaf(qv.w, e[x + 3], acc[gg]);
+              }
             }
           }
         }
       }
-    }
 #pragma unroll
-    for (int gg = 0; gg < G; ++gg) acc[gg] += __shfl_xor_sync(0xffffffffu, acc[gg], 1);
-    if (ok && half == 0) {
+      for (int gg = 0; gg < G; ++gg) acc[gg] += __shfl_xor_sync(0xffffffffu, acc[gg], 1);
+      if (ok && half == 0) {
 #pragma unroll
-      for (int gg = 0; gg < G; ++gg) zbuf[kk * ldz + g * G + gg] = acc[gg];
+        for (int gg = 0; gg < G; ++gg) zbuf[kk * ldz + g * G + gg] = acc[gg];
+      }
     }
-  }
-  __syncthreads();
+    __syncthreads();
 
-  // per-head chunk statistics: max, sums of 2^(z - max) over all and over visual keys
-  const int vlo = max(p_begin, v0), vhi = min(p_begin + nk, v0 + nvis);
-  for (int h = warp; h < Hq; h += kScoreThreads / 32) {
-    float mx = -INFINITY;
-    for (int kk = lane; kk < nk; kk += 32) mx = fmaxf(mx, zbuf[kk * ldz + h]);
+    // per-head chunk statistics: max, sums of 2^(z - max) over all and over visual keys
+    const int vlo = max(p_begin, v0), vhi = min(p_begin + nk, v0 + nvis);
+    for (int h = warp; h < Hq; h += kScoreThreads / 32) {
+      float mx = -INFINITY;
+      for (int kk = lane; kk < nk; kk += 32) mx = fmaxf(mx, zbuf[kk * ldz + h]);
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-    float sum = 0.f, vis = 0.f;
-    for (int kk = lane; kk < nk; kk += 32) {
-      const float e = exp2f(zbuf[kk * ldz + h] - mx);
-      sum += e;
-      const int p = p_begin + kk;
-      if (p >= vlo && p < vhi) vis += e;
-    }
+      for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+      float sum = 0.f, vis = 0.f;
+      for (int kk = lane; kk < nk; kk += 32) {
+        const float e = exp2f(zbuf[kk * ldz + h] - mx);
+        sum += e;
+        const int p = p_begin + kk;
+        if (p >= vlo && p < vhi) vis += e;
+      }
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      sum += __shfl_xor_sync(0xffffffffu, sum, o);
-      vis += __shfl_xor_sync(0xffffffffu, vis, o);
+      for (int o = 16; o > 0; o >>= 1) {
+        sum += __shfl_xor_sync(0xffffffffu, sum, o);
+        vis += __shfl_xor_sync(0xffffffffu, vis, o);
+      }
+      if (lane == 0)
+        a.stats[((long long)l * Hq + h) * a.total_chunks + cbase + chunk] =
+            make_float4(mx, sum, vis, 0.f);
     }
-    if (lane == 0)
-      a.stats[((long long)l * Hq + h) * a.total_chunks + cbase + chunk] =
-          make_float4(mx, sum, vis, 0.f);
-  }
 
-  // visual logits of this chunk
-  const int nv = vhi - vlo;
-  if (nv > 0) {
-    for (int idx = tid; idx < nv * Hq; idx += kScoreThreads) {
-      const int h = idx / nv, i = idx - h * nv;
-      const int p = vlo + i;
-      a.zlog[((long long)l * Hq + h) * a.total_vis + voff + (p - v0)] =
-          zbuf[(p - p_begin) * ldz + h];
+    // visual logits of this chunk
+    const int nv = vhi - vlo;
+    if (nv > 0) {
+      for (int idx = tid; idx < nv * Hq; idx += kScoreThreads) {
+        const int h = idx / nv, i = idx - h * nv;
+        const int p = vlo + i;
+        a.zlog[((long long)l * Hq + h) * a.total_vis + voff + (p - v0)] =
+            zbuf[(p - p_begin) * ldz + h];
+      }
     }
   }
+  // the token kernel (launched as a programmatic dependent) may start its
+  // prologue; it waits for this whole grid before reading any result
+  asm volatile("griddepcontrol.launch_dependents;");
 }
 
 // Eq. 7-8: one CTA per (request b, tile of kTokenTile visual tokens).
@@ -167,6 +197,9 @@ score_tokens_kernel(const ScoreArgs a) {
   const int32_t *m = a.meta + b * kMetaFields;
   const int nvis = m[kNumVis], voff = m[kVisOff], cbase = m[kChunkBase];
   if (tile * kTokenTile >= nvis) return;
+  // launched as a programmatic dependent of score_logits_kernel: wait until that
+  // grid has completed and its writes are visible (a no-op for a plain launch)
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   const int nch = (m[kSeqLen] + a.chunk - 1) / a.chunk;
   const int LH = a.L * a.Hq;
   float *cmax = coef, *cinv = coef + LH, *cvis = coef + 2 * LH;
@@ -249,6 +282,30 @@ size_t logits_smem(const Plan &pl) {
 
 constexpr size_t kMaxScoreSmem = 100 * 1024;
 
+// CTAs of `fn` resident on the whole current device (occupancy x SMs), cached
+// per (device, kernel, shared memory).
+cudaError_t resident_slots(const void *fn, size_t smem, int *slots) {
+  static std::mutex mu;
+  static std::map<std::tuple<int, const void *, size_t>, int> cache;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const auto key = std::make_tuple(dev, fn, smem);
+  std::lock_guard<std::mutex> lock(mu);
+  auto hit = cache.find(key);
+  if (hit != cache.end()) {
+    *slots = hit->second;
+    return cudaSuccess;
+  }
+  int per_sm = 0, sms = 0;
+  if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, kScoreThreads, smem)) != cudaSuccess)
+    return e;
+  if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
+  *slots = std::max(per_sm, 1) * sms;
+  cache.emplace(key, *slots);
+  return cudaSuccess;
+}
+
 }  // namespace
 
 int score_chunk_keys(int num_kv_heads) {
@@ -298,8 +355,12 @@ cudaError_t launch_scores(const Plan &pl, const void *q, const void *k, float *w
     e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
   }
+  int slots = 0;
+  if ((e = resident_slots(fn, smem, &slots)) != cudaSuccess) return e;
+  const long long items = (long long)pl.total_chunks * pl.L;
+  const int grid = (int)std::min<long long>(items, slots);
   void *args[] = {&a};
-  e = cudaLaunchKernel(fn, dim3(pl.total_chunks, pl.L), dim3(kScoreThreads), args, smem, s);
+  e = cudaLaunchKernel(fn, dim3(grid), dim3(kScoreThreads), args, smem, s);
   if (e != cudaSuccess) return e;
   const int max_tiles = (pl.max_vis + kTokenTile - 1) / kTokenTile;
   const size_t tsmem = sizeof(float) * 3 * pl.L * pl.Hq;
@@ -308,7 +369,18 @@ cudaError_t launch_scores(const Plan &pl, const void *q, const void *k, float *w
                              (int)tsmem);
     if (e != cudaSuccess) return e;
   }
-  score_tokens_kernel<<<dim3(max_tiles, pl.B), kScoreThreads, tsmem, s>>>(a);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(max_tiles, pl.B);
+  cfg.blockDim = dim3(kScoreThreads);
+  cfg.dynamicSmemBytes = tsmem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  e = cudaLaunchKernelEx(&cfg, score_tokens_kernel, a);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 

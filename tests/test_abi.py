@@ -81,6 +81,29 @@ def test_select_rejects_bad_problems_before_launch(lib, kw, status):
     assert e.value.status == status
 
 
+@pytest.mark.parametrize("kw,args,status", [
+    (dict(cu_keep=[0, 7, 9]), dict(x=16, x_out=16), last.LAST_ERR_INVALID_ARG),     # k_b > N_b
+    (dict(feat_dim=100), dict(x=16, x_out=16), last.LAST_ERR_INVALID_ARG),          # gather width
+    (dict(), dict(x=None, x_out=16), last.LAST_ERR_INVALID_ARG),                    # x missing
+    (dict(), dict(x=24, x_out=16), last.LAST_ERR_INVALID_ARG),                      # misaligned x
+])
+def test_topk_rejects_bad_arguments_before_launch(lib, kw, args, status):
+    prob = _problem(**kw)
+    with pytest.raises(last.LastError) as e:
+        last.last_select_topk(prob, 16, 16, (256, 1 << 30), stream=0, **args)
+    assert e.value.status == status
+
+
+def test_topk_needs_no_sequence_fields(lib):
+    # scores-only fields may be absent; validation then fails only on the workspace
+    prob = last.Problem(batch=1, num_layers=0, num_q_heads=0, num_kv_heads=0, head_dim=0,
+                        feat_dim=8, dtype="bf16", cu_seqlens=None, vis_start=None,
+                        cu_vis=[0, 5], cu_keep=[0, 2])
+    with pytest.raises(last.LastError) as e:
+        last.last_select_topk(prob, 16, 16, (256, 1), stream=0)
+    assert e.value.status == last.LAST_ERR_WORKSPACE_TOO_SMALL
+
+
 def test_workspace_checks(lib):
     prob = _problem()
     need = last.last_workspace_size(prob)
