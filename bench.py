@@ -414,7 +414,7 @@ def main():
                     "scores_GBps": sc_gbs, "scores_hbm_frac": sc_gbs / hbm},
         "roofline": {"bound": "alu", "kernel": "select_kernel", "achieved": achieved,
                      "peak": alu_peak_tflops, "unit": "TFLOP/s", "frac": achieved / alu_peak_tflops,
-                     "traffic": measured_traffic("select_kernels.cu",
+                     "traffic": measured_traffic("select_impl.cuh",
                                                  f"{args.workload}-{args.budget}"),
                      "peak_note": f"{sm_count} SMs x {FP32_LANES_PER_SM} fp32 FMA/clk x 2 x "
                                   f"{sm_max:.0f} MHz ({pk_kind} max clock)"},

@@ -312,6 +312,9 @@ last_status last_poll(const void *ws, void *stream) {
   cudaError_t e = cudaMemcpyAsync(&flag, ws, sizeof flag, cudaMemcpyDeviceToHost, s);
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
   if (e != cudaSuccess) return cuda_fail(e, "poll");
+  if (flag & kErrConfig)
+    return fail(LAST_ERR_CUDA, "internal error: a kernel's shared-memory plan exceeded its launch; "
+                               "outputs of that call are invalid");
   if (flag & kErrTimeout)
     return fail(LAST_ERR_TIMEOUT, "a bounded device wait expired; outputs of that call are invalid");
   if (flag & kErrGatherIndex)

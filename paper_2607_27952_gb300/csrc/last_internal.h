@@ -34,6 +34,7 @@ constexpr int kGatherThreads = 256;
 // Device error flags (first word of the workspace).
 constexpr unsigned kErrGatherIndex = 1u;
 constexpr unsigned kErrTimeout = 2u;      // a bounded wait on a bulk copy expired
+constexpr unsigned kErrConfig = 4u;       // a kernel's shared-memory plan exceeded its launch
 
 struct Plan {
   // problem
