@@ -55,8 +55,8 @@ constexpr int kRing = 4;                           // async-copy ring depth (gro
 // Tensor-core update (bf16): 128-row tiles of X against up to 16 new centres.
 constexpr int kTcBM = 128, kTcBK = 64;             // MMA M; K elements per 128-byte row
                                                    // (MMA N = the candidate list length)
-constexpr int kTcStages = 4;                       // TMA ring depth
-constexpr int kTcStageBytes = kTcBM * kTcBK * 2;   // one A box: 16 KB
+constexpr int kTcMaxStages = 12;                   // TMA ring depth (runtime a.tc_stages)
+constexpr int kTcBoxBytes = kTcBM * kTcBK * 2;     // one A box (128 rows x 64 elements): 16 KB
 constexpr int kTmemCols = 512;                     // TMEM columns per SM
 
 struct SelectArgs {
@@ -73,6 +73,8 @@ struct SelectArgs {
   int lcap;              // candidate list length (16 or 32)
   unsigned *err;         // workspace error word
   uint32_t tmem_cols;    // tc: TMEM columns allocated (power of two >= 32)
+  int tc_stages;         // tc: TMA ring depth (2..kTcMaxStages)
+  int tc_kps;            // tc: K blocks (boxes) per ring stage
   float tc_eps;          // tc: bound on |tensor-core distance - canonical distance|
 };
 
@@ -94,7 +96,7 @@ __host__ __device__ inline int blocks_per_warp(int tpc_max, int tb) {
 }
 __host__ __device__ inline SelectSmem select_smem(int cache_rows, int row_bytes, int tpc_max,
                                                   int ring, int tb, int elem, int lcap,
-                                                  int tc = 0) {
+                                                  int tc = 0, int stages = 0, int kps = 1) {
   SelectSmem s;
   size_t o = 0;
   if (tc) {
@@ -102,7 +104,7 @@ __host__ __device__ inline SelectSmem select_smem(int cache_rows, int row_bytes,
     // K block kb of list row j at kb * lcap * 128 + j * 128; both regions are
     // multiples of 1024 bytes from a 1024-aligned base
     s.cbuf = o; o += (size_t)tc_kblocks(row_bytes / elem) * lcap * 128;
-    s.aring = o; o += (size_t)kTcStages * kTcStageBytes;
+    s.aring = o; o += (size_t)stages * kps * kTcBoxBytes;
     s.xcache = o;
     s.ring = o;
     s.blk = o;
@@ -131,7 +133,7 @@ __host__ __device__ inline SelectSmem select_smem(int cache_rows, int row_bytes,
   s.bar = o; o += sizeof(unsigned long long);
   s.cnt = o; o += sizeof(int) * kMaxCluster;
   o = align16(o);
-  s.tbar = o; o += tc ? sizeof(unsigned long long) * (2 * kTcStages + 1) : 0;
+  s.tbar = o; o += tc ? sizeof(unsigned long long) * (2 * kTcMaxStages + 1) : 0;
   s.tslot = o; o += tc ? 16 : 0;
   s.fidx = o; o += tc ? align16(sizeof(int) * tpc_max) : 0;
   s.fmask = o; o += tc ? align16(sizeof(unsigned short) * tpc_max) : 0;
@@ -227,7 +229,7 @@ select_kernel(const __grid_constant__ SelectArgs a) {
   if (K == 0) return;  // the whole cluster leaves together; no DSMEM traffic yet
 
   const SelectSmem S = select_smem(a.cache_rows, a.row_bytes, a.tpc_max, a.ring, TB, (int)sizeof(T),
-                                   a.lcap, TC ? 1 : 0);
+                                   a.lcap, TC ? 1 : 0, TC ? a.tc_stages : 0, TC ? a.tc_kps : 1);
   {
     // The host sizes the launch with the same plan; should they ever disagree, every
     // CTA of every cluster leaves here together (before any cluster barrier)
@@ -276,12 +278,13 @@ select_kernel(const __grid_constant__ SelectArgs a) {
   // parity of the next phase to wait for.
   uint32_t phase = 0;
   unsigned long long *tfull = reinterpret_cast<unsigned long long *>(smem + S.tbar);
-  unsigned long long *tempty = tfull + kTcStages;
-  unsigned long long *tdone = tempty + kTcStages;
+  const int nstage = TC ? a.tc_stages : 1;
+  unsigned long long *tempty = tfull + kTcMaxStages;
+  unsigned long long *tdone = tempty + kTcMaxStages;
   if (threadIdx.x == 0) {
     mbar_init(bar, 1);
     if constexpr (TC) {
-      for (int i = 0; i < kTcStages; ++i) {
+      for (int i = 0; i < nstage; ++i) {
         mbar_init(&tfull[i], 1);
         mbar_init(&tempty[i], 1);
       }
@@ -630,30 +633,41 @@ select_kernel(const __grid_constant__ SelectArgs a) {
       tc_fence_after();
       // 2. TMA producer (thread 0) and MMA issuer (thread 32)
       const int ntile = (nloc + kTcBM - 1) / kTcBM;
+      // a ring stage holds kps consecutive K blocks of one tile (one barrier, one
+      // commit): the per-stage hand-off costs the same whatever the stage size
+      const int kps = a.tc_kps;
+      const int stage_bytes = kps * kTcBoxBytes;
+      const int ngrp = (nkb + kps - 1) / kps;
       if (threadIdx.x == 0) {
         for (int tile = 0; tile < ntile; ++tile)
-          for (int kb = 0; kb < nkb; ++kb, ++tc_pit) {
-            const int st = tc_pit % kTcStages;
-            if (tc_pit >= kTcStages && !twait(&tempty[st], ((tc_pit / kTcStages) - 1) & 1))
-              continue;   // expired: the box is skipped and the call reports the timeout
-            mbar_expect_tx(&tfull[st], kTcStageBytes);
-            tma_load_2d(aring + st * kTcStageBytes, &a.tmap, kb * kTcBK, voff + lo + tile * kTcBM,
-                        &tfull[st]);
+          for (int gq = 0; gq < ngrp; ++gq, ++tc_pit) {
+            const int st = tc_pit % nstage;
+            if (tc_pit >= (uint32_t)nstage && !twait(&tempty[st], ((tc_pit / nstage) - 1) & 1))
+              continue;   // expired: the stage is skipped and the call reports the timeout
+            const int nb = min(kps, nkb - gq * kps);
+            mbar_expect_tx(&tfull[st], (uint32_t)(nb * kTcBoxBytes));
+            for (int q = 0; q < nb; ++q)
+              tma_load_2d(aring + st * stage_bytes + q * kTcBoxBytes, &a.tmap, (gq * kps + q) * kTcBK,
+                          voff + lo + tile * kTcBM, &tfull[st]);
           }
       } else if (threadIdx.x == 32) {
         const uint32_t idesc = umma_idesc_bf16(kTcBM, lcap);
         for (int tile = 0; tile < ntile; ++tile)
-          for (int kb = 0; kb < nkb; ++kb, ++tc_mit) {
-            const int st = tc_mit % kTcStages;
-            const bool ok = twait(&tfull[st], (tc_mit / kTcStages) & 1);
+          for (int gq = 0; gq < ngrp; ++gq, ++tc_mit) {
+            const int st = tc_mit % nstage;
+            const bool ok = twait(&tfull[st], (tc_mit / nstage) & 1);
             tc_fence_after();
             if (ok) {
+              const int nb = min(kps, nkb - gq * kps);
+              for (int q = 0; q < nb; ++q) {
+                const int kb = gq * kps + q;
 #pragma unroll
-              for (int k = 0; k < kTcBK / 16; ++k)
-                umma_bf16(tmem + tile * lcap,
-                          umma_desc_sw128(smem_addr(aring + st * kTcStageBytes) + k * 32),
-                          umma_desc_sw128(cbuf_sa + kb * lcap * 128 + k * 32), idesc,
-                          (kb | k) != 0 ? 1u : 0u);
+                for (int k = 0; k < kTcBK / 16; ++k)
+                  umma_bf16(tmem + tile * lcap,
+                            umma_desc_sw128(smem_addr(aring + st * stage_bytes + q * kTcBoxBytes) + k * 32),
+                            umma_desc_sw128(cbuf_sa + kb * lcap * 128 + k * 32), idesc,
+                            (kb | k) != 0 ? 1u : 0u);
+              }
             }
             umma_commit(&tempty[st]);   // frees the stage once these MMAs have read it
           }
@@ -699,18 +713,10 @@ select_kernel(const __grid_constant__ SelectArgs a) {
       }
       tc_fence_before();
       __syncthreads();
-      // 4. exact canonical distances for the flagged pairs (a warp per token)
+      // 4. exact canonical distances for the flagged pairs (a warp per token, two
+      //    tokens' rows in flight)
       const int nf = *fcnt;
-      for (int f = warp; f < nf; f += kSelectWarps) {
-        const int t = fidx[f];
-        unsigned msk = fmask[f];
-        const char *xrow = xg + (long long)t * rb;
-        U4 xv[NCH];
-#pragma unroll
-        for (int g = 0; g < NCH; ++g) {
-          const int col = 256 * g + 8 * lane;
-          xv[g] = col < dv ? ldg(xrow + col * 2) : U4{0, 0, 0, 0};
-        }
+      auto exact_token = [&](int t, unsigned msk, const U4 *xv) {
         const float ri = r_s[t];
         float dl = dl_s[t];
         while (msk) {
@@ -736,6 +742,19 @@ select_kernel(const __grid_constant__ SelectArgs a) {
           dl = fminf(dl, __fsub_rn(1.0f, __fmul_rn(__fmul_rn(dot, ri), lp_f[acc_s[j] * 3 + 2])));
         }
         if (lane == 0) dl_s[t] = dl;
+      };
+      for (int f = warp; f < nf; f += 2 * kSelectWarps) {
+        const int f2 = f + kSelectWarps;
+        const int t0 = fidx[f], t1 = f2 < nf ? fidx[f2] : t0;
+        U4 xa[NCH], xb[NCH];
+#pragma unroll
+        for (int g = 0; g < NCH; ++g) {
+          const int col = 256 * g + 8 * lane;
+          xa[g] = col < dv ? ldg(xg + (long long)t0 * rb + col * 2) : U4{0, 0, 0, 0};
+          xb[g] = col < dv ? ldg(xg + (long long)t1 * rb + col * 2) : U4{0, 0, 0, 0};
+        }
+        exact_token(t0, fmask[f], xa);
+        if (f2 < nf) exact_token(t1, fmask[f2], xb);
       }
       __syncthreads();
       // 5. keys of the unselected tokens -> the warp's ranked list for the next round

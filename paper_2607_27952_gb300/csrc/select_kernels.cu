@@ -29,15 +29,35 @@ void *pick_select(int dtype, int nch, int tb, bool tc) {
 struct DeviceInfo {
   int optin = 0, sms = 0;
   double l2 = 0.0;
+  double dram_bytes_per_cycle = 0.0;   // sustained DRAM bytes per SM clock, whole device
 };
+// Queried once per device: some attributes (clock rates) are slow to read.
 DeviceInfo device_info() {
-  DeviceInfo d;
-  int dev = 0, v = 0;
+  static std::mutex mu;
+  static std::map<int, DeviceInfo> cache;
+  int dev = 0;
   cudaGetDevice(&dev);
+  {
+    std::lock_guard<std::mutex> lock(mu);
+    auto hit = cache.find(dev);
+    if (hit != cache.end()) return hit->second;
+  }
+  DeviceInfo d;
+  int v = 0, mem_khz = 0, bus_bits = 0, sm_khz = 0;
   cudaDeviceGetAttribute(&d.optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
   cudaDeviceGetAttribute(&d.sms, cudaDevAttrMultiProcessorCount, dev);
   cudaDeviceGetAttribute(&v, cudaDevAttrL2CacheSize, dev);
+  cudaDeviceGetAttribute(&mem_khz, cudaDevAttrMemoryClockRate, dev);
+  cudaDeviceGetAttribute(&bus_bits, cudaDevAttrGlobalMemoryBusWidth, dev);
+  cudaDeviceGetAttribute(&sm_khz, cudaDevAttrClockRate, dev);
   d.l2 = v;
+  // double data rate; about 80% of the nominal rate is sustained
+  if (mem_khz > 0 && bus_bits > 0 && sm_khz > 0)
+    d.dram_bytes_per_cycle = 0.8 * 2.0 * mem_khz * (bus_bits / 8.0) / sm_khz;
+  else
+    d.dram_bytes_per_cycle = 3000.0;
+  std::lock_guard<std::mutex> lock(mu);
+  cache.emplace(dev, d);
   return d;
 }
 
@@ -147,7 +167,7 @@ cudaError_t launch_select(const Plan &pl, const float *w, const void *x, int32_t
   //   waves x (one round's update + round overhead)
   // (the round count of a request does not depend on C to first order); small
   // clusters raise the number of requests in flight, large ones shorten each round.
-  int C = 0, tpc = 0, cache_rows = 0, ring = 0, lcap = kLcap / 2;
+  int C = 0, tpc = 0, cache_rows = 0, ring = 0, lcap = kLcap / 2, stages = 0, kps = 1;
   size_t smem = 0;
   double best = 0.0;
   void *fn = nullptr;
@@ -157,14 +177,23 @@ cudaError_t launch_select(const Plan &pl, const float *w, const void *x, int32_t
     // 2 for fp32 and the tensor-core update, else 4 unless a CTA owns few tokens
     const int tb_c = (pl.elem == 4 || tc || tpc_c < 64) ? 2 : 4;
     void *fn_c = pick_select(pl.dtype, nch, tb_c, tc);
-    int cache_c = 0, ring_c = 0, lcap_c = 0;
+    int cache_c = 0, ring_c = 0, lcap_c = 0, stages_c = 0, kps_c = 1;
     size_t smem_c = 0;
     if (tc) {
-      // the list length is the MMA N: lcap accumulator columns per 128-row tile
+      // the list length is the MMA N: lcap accumulator columns per 128-row tile; the
+      // TMA ring takes the shared memory left over
       const int tiles = (tpc_c + kTcBM - 1) / kTcBM;
+      // stages of kps boxes: the largest kps (<= 4) that still leaves 2 stages
       for (int lc = (c <= 4 ? kLcap : kLcap / 2); lc >= kLcap / 2 && lcap_c == 0; lc /= 2) {
-        const size_t sz = select_smem(0, rb, tpc_c, 0, tb_c, pl.elem, lc, 1).total;
-        if (sz <= (size_t)di.optin && tiles * lc <= kTmemCols) { lcap_c = lc; smem_c = sz; }
+        const size_t fixed = select_smem(0, rb, tpc_c, 0, tb_c, pl.elem, lc, 1, 0).total;
+        if (fixed + 2 * (size_t)kTcBoxBytes > (size_t)di.optin || tiles * lc > kTmemCols) continue;
+        const size_t room = di.optin - fixed;
+        kps_c = 1;
+        while (kps_c < 4 && room >= 2 * (size_t)(2 * kps_c) * kTcBoxBytes) kps_c *= 2;
+        kps_c = std::min(kps_c, tc_kblocks(pl.dv));
+        stages_c = (int)std::min<size_t>(kTcMaxStages, room / ((size_t)kps_c * kTcBoxBytes));
+        lcap_c = lc;
+        smem_c = select_smem(0, rb, tpc_c, 0, tb_c, pl.elem, lc, 1, stages_c, kps_c).total;
       }
       if (lcap_c == 0) continue;
     } else {
@@ -189,9 +218,15 @@ cudaError_t launch_select(const Plan &pl, const float *w, const void *x, int32_t
     const bool from_hbm = in_flight > 0.7 * di.l2;
     double round_cycles;
     if (tc) {
-      // the update streams this CTA's rows (whole 128-row tiles) once per round
+      // The update streams this CTA's rows (whole 128-row tiles) once per round, at
+      // the smaller of the ring's hand-off rate (about 900 cycles per stage, measured)
+      // and this CTA's share of DRAM (or of L2, taken as 2.5x, when the features of
+      // the requests in flight fit in it).
       const double bytes = (double)((tpc_c + kTcBM - 1) / kTcBM) * kTcBM * tc_kblocks(pl.dv) * 128.0;
-      round_cycles = bytes / (from_hbm ? 20.0 : 48.0) + 12000.0 + 400.0 * c;
+      const double ctas = std::min<double>(pl.B, active) * c;
+      const double share = di.dram_bytes_per_cycle / ctas * (from_hbm ? 1.0 : 2.5);
+      const double bw = std::min(kps_c * (double)kTcBoxBytes / 900.0, share);
+      round_cycles = bytes / bw + 30000.0 + 400.0 * c;
     } else {
       const double stream_penalty = from_hbm ? 3.0 : 1.0;
       const double streamed = std::max(0, tpc_c - cache_c), cached = std::min(tpc_c, cache_c);
@@ -200,7 +235,7 @@ cudaError_t launch_select(const Plan &pl, const float *w, const void *x, int32_t
     const double cost = waves * round_cycles;
     if (C == 0 || cost < best) {
       best = cost; C = c; tpc = tpc_c; cache_rows = cache_c; smem = smem_c; ring = ring_c;
-      lcap = lcap_c; fn = fn_c;
+      lcap = lcap_c; fn = fn_c; stages = stages_c; kps = kps_c;
     }
   }
   if (C == 0) return cudaErrorInvalidConfiguration;
@@ -223,6 +258,8 @@ cudaError_t launch_select(const Plan &pl, const float *w, const void *x, int32_t
     uint32_t tcols = 32;
     while ((int)tcols < cols) tcols *= 2;
     a.tmem_cols = tcols;
+    a.tc_stages = stages;
+    a.tc_kps = kps;
     a.tc_eps = tc_distance_eps(pl.dv);
   }
 
