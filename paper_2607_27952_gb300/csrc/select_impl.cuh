@@ -47,8 +47,11 @@ namespace last {
 constexpr int kSelThreads = kSelectWarps * 32;
 constexpr int kMaxCluster = 16;
 constexpr int kLcap = 32;                          // candidate list capacity (runtime a.lcap <= kLcap)
-constexpr int kMaxAccept = 16;                     // picks folded into delta per round
-constexpr int kTopM = 9;                           // per-warp / per-CTA ranked keys (<= 8 + bound)
+constexpr int kMaxAccept = 32;                     // picks folded into delta per round (runtime a.max_accept)
+constexpr int kTopMax = 17;                        // ranked keys per warp / CTA: <= 16 published + bound
+// ranked keys the kernel keeps: 8 + bound on the CUDA-core update (register
+// budget), 16 + bound with the tensor-core update
+template <bool TC> __host__ __device__ constexpr int top_width() { return TC ? 17 : 9; }
 constexpr int kMaxPairs = kLcap * (kLcap - 1) / 2;
 constexpr int kRing = 4;                           // async-copy ring depth (groups in flight)
 
@@ -68,7 +71,8 @@ struct SelectArgs {
   const int32_t *meta;
   const int32_t *order;  // cluster -> request (most work first)
   int dv, row_bytes, tpc_max, cache_rows, csize;
-  int mc;                // candidates each CTA publishes per round (<= kTopM - 1)
+  int mc;                // candidates each CTA publishes per round (< top_width)
+  int max_accept;        // picks accepted per round (<= kMaxAccept; 16 on the CUDA-core update)
   int ring;              // 1: rows beyond the resident cache stream through an async-copy ring
   int lcap;              // candidate list length (16 or 32)
   unsigned *err;         // workspace error word
@@ -120,23 +124,23 @@ __host__ __device__ inline SelectSmem select_smem(int cache_rows, int row_bytes,
   s.dl = o; o += align16(sizeof(float) * tpc_max);
   s.list = o; o += align16(sizeof(int) * tpc_max);
   s.sel = o; o += align16(tpc_max);
-  s.wtop = o; o += sizeof(unsigned long long) * kSelectWarps * kTopM;
-  s.pub_key = o; o += sizeof(unsigned long long) * 2 * kMaxCluster * kTopM;
-  s.pub_f = o; o += sizeof(float4) * 2 * kMaxCluster * kTopM;
+  s.wtop = o; o += sizeof(unsigned long long) * kSelectWarps * kTopMax;
+  s.pub_key = o; o += sizeof(unsigned long long) * 2 * kMaxCluster * kTopMax;
+  s.pub_f = o; o += sizeof(float4) * 2 * kMaxCluster * kTopMax;
   s.lp_key = o; o += sizeof(unsigned long long) * kLcap;
   s.lp_f = o; o += sizeof(float) * kLcap * 3;
   s.lp_idx = o; o += sizeof(int) * kLcap;
   s.lp_row = o; o += sizeof(int) * kLcap;
   s.pair = o; o += sizeof(float) * 2 * kMaxPairs;
   s.acc = o; o += sizeof(int) * kMaxAccept;
-  s.misc = o; o += sizeof(unsigned long long) * (4 + kTopM);
+  s.misc = o; o += sizeof(unsigned long long) * (4 + kTopMax);
   s.bar = o; o += sizeof(unsigned long long);
   s.cnt = o; o += sizeof(int) * kMaxCluster;
   o = align16(o);
   s.tbar = o; o += tc ? sizeof(unsigned long long) * (2 * kTcMaxStages + 1) : 0;
   s.tslot = o; o += tc ? 16 : 0;
   s.fidx = o; o += tc ? align16(sizeof(int) * tpc_max) : 0;
-  s.fmask = o; o += tc ? align16(sizeof(unsigned short) * tpc_max) : 0;
+  s.fmask = o; o += tc ? align16(sizeof(uint32_t) * tpc_max) : 0;
   s.fcnt = o; o += tc ? 16 : 0;
   s.total = align16(o) + 1024;   // slack for aligning the base to 1024 bytes
   return s;
@@ -196,17 +200,18 @@ __device__ __forceinline__ void warp_argmax(unsigned long long &key, int &payloa
   }
 }
 
-// descending top-kTopM list held in (warp-uniform) registers
+// descending top-W list held in (warp-uniform) registers
+template <int W>
 struct TopList {
-  unsigned long long k[kTopM];
+  unsigned long long k[W];
   __device__ __forceinline__ void clear() {
 #pragma unroll
-    for (int i = 0; i < kTopM; ++i) k[i] = 0ull;
+    for (int i = 0; i < W; ++i) k[i] = 0ull;
   }
   __device__ __forceinline__ void insert(unsigned long long v) {
-    if (v <= k[kTopM - 1]) return;
+    if (v <= k[W - 1]) return;
 #pragma unroll
-    for (int i = kTopM - 1; i > 0; --i) {
+    for (int i = W - 1; i > 0; --i) {
       if (v > k[i - 1]) k[i] = k[i - 1];
       else if (v > k[i]) { k[i] = v; v = 0ull; }
     }
@@ -217,6 +222,7 @@ struct TopList {
 template <typename T, int NCH, int TB, bool TC>
 __global__ void __launch_bounds__(kSelThreads, 1)
 select_kernel(const __grid_constant__ SelectArgs a) {
+  constexpr int kTop = top_width<TC>();
   extern __shared__ __align__(16) unsigned char smem_raw[];
   unsigned char *smem = reinterpret_cast<unsigned char *>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -325,7 +331,7 @@ select_kernel(const __grid_constant__ SelectArgs a) {
       tmem = *tslot;
     }
     // r_i = 1/sqrt(dot(x_i, x_i)); each warp also ranks its tokens by w~ for the seed
-    TopList top;
+    TopList<kTop> top;
     top.clear();
     for (int t = warp; t < nloc; t += kSelectWarps) {
       const bool sh = t < ncache;
@@ -336,18 +342,18 @@ select_kernel(const __grid_constant__ SelectArgs a) {
     }
     if (lane == 0) {
 #pragma unroll
-      for (int i = 0; i < kTopM; ++i) wtop[warp * kTopM + i] = top.k[i];
+      for (int i = 0; i < kTop; ++i) wtop[warp * kTop + i] = top.k[i];
     }
     __syncthreads();
 
-    // Merge the warps' lists into the CTA's kTopM best and publish them (key and
+    // Merge the warps' lists into the CTA's kTop best and publish them (key and
     // {delta, w, r}) to every CTA of the cluster, into buffer `par`.
-    unsigned long long *top5 = misc + 4;  // misc[4..4+kTopM)
+    unsigned long long *top5 = misc + 4;  // misc[4..4+kTop)
     auto publish = [&](int par) {
       if (warp == 0) {
-        constexpr int nk = kSelectWarps * kTopM;   // the warps' ranked keys
+        constexpr int nk = kSelectWarps * kTop;   // the warps' ranked keys
         constexpr int kPerLane = (nk + 31) / 32;
-        static_assert(kPerLane <= 3, "publish ranks at most 96 keys");
+        static_assert(kPerLane <= 5, "publish ranks at most 160 keys");
         unsigned long long kl[kPerLane];
         int rl[kPerLane];
 #pragma unroll
@@ -355,7 +361,7 @@ select_kernel(const __grid_constant__ SelectArgs a) {
           kl[j] = lane + 32 * j < nk ? wtop[lane + 32 * j] : 0ull;
           rl[j] = 0;
         }
-        if (lane < kTopM) top5[lane] = 0ull;
+        if (lane < kTop) top5[lane] = 0ull;
 #pragma unroll
         for (int f = 0; f < nk; ++f) {
           const unsigned long long kf = wtop[f];
@@ -365,12 +371,12 @@ select_kernel(const __grid_constant__ SelectArgs a) {
         __syncwarp();
 #pragma unroll
         for (int j = 0; j < kPerLane; ++j)
-          if (kl[j] != 0ull && rl[j] < kTopM) top5[rl[j]] = kl[j];
+          if (kl[j] != 0ull && rl[j] < kTop) top5[rl[j]] = kl[j];
         __syncwarp();
         if (lane < C) {
           for (int i = 0; i <= a.mc; ++i) {
             const unsigned long long key = top5[i];
-            const int slot = (par * kMaxCluster + (int)rank) * kTopM + i;
+            const int slot = (par * kMaxCluster + (int)rank) * kTopMax + i;
             float4 f = make_float4(0.f, 0.f, 0.f, 0.f);
             if (key != 0ull) {
               const int lt = key_index(key) - lo;
@@ -492,7 +498,7 @@ select_kernel(const __grid_constant__ SelectArgs a) {
       };
       if (streams)
         for (int i = 0; i < kRing - 1; ++i) issue();
-      TopList tl;
+      TopList<kTop> tl;
       tl.clear();
       uint32_t cslot = 0;       // ring slot of the item being computed
       for (int j = 0; j < nact; ++j) {
@@ -595,7 +601,7 @@ select_kernel(const __grid_constant__ SelectArgs a) {
       cp_async_wait<0>();
       if (lane == 0) {
 #pragma unroll
-        for (int i = 0; i < kTopM; ++i) wtop[warp * kTopM + i] = tl.k[i];
+        for (int i = 0; i < kTop; ++i) wtop[warp * kTop + i] = tl.k[i];
       }
     };
     // Tensor-core form of the same update (bf16).  X's rows of this CTA stream
@@ -622,7 +628,7 @@ select_kernel(const __grid_constant__ SelectArgs a) {
       const int nkb = tc_kblocks(dv);
       char *aring = reinterpret_cast<char *>(smem + S.aring);
       int *fidx = reinterpret_cast<int *>(smem + S.fidx);
-      unsigned short *fmask = reinterpret_cast<unsigned short *>(smem + S.fmask);
+      uint32_t *fmask = reinterpret_cast<uint32_t *>(smem + S.fmask);
       int *fcnt = reinterpret_cast<int *>(smem + S.fcnt);
       // 1. the B operand is cbuf as staged (every list row; the accepted centres are
       //    the accumulator columns lp_row[acc_s[j]])
@@ -679,36 +685,32 @@ select_kernel(const __grid_constant__ SelectArgs a) {
       tc_fence_after();
       // 3. certify: flag (token, centre) pairs the tensor-core distance cannot decide
       const float eps = a.tc_eps;
-      float rc[kMaxAccept];
-      int col[kMaxAccept];
-#pragma unroll
-      for (int j = 0; j < kMaxAccept; ++j) {
-        rc[j] = j < nA ? lp_f[acc_s[j] * 3 + 2] : 0.f;
-        col[j] = j < nA ? lp_row[acc_s[j]] : 0;
-      }
       for (int tt = warp >> 2; tt < ntile; tt += 2) {
-        uint32_t dv_[kMaxAccept];
         const uint32_t tbase = tmem + ((uint32_t)(32 * (warp & 3)) << 16) + (uint32_t)(tt * lcap);
-#pragma unroll
-        for (int j = 0; j < kMaxAccept; ++j)
-          if (j < nA) tmem_ld1(tbase + (uint32_t)col[j], &dv_[j]);
-        tmem_wait_ld();
         const int t = tt * kTcBM + 32 * (warp & 3) + lane;
-        if (t < nloc && !sel_s[t]) {
-          const float ri = r_s[t], dl = dl_s[t];
-          unsigned msk = 0;
+        const bool live = t < nloc && !sel_s[t];
+        const float ri = live ? r_s[t] : 0.f, dl = live ? dl_s[t] : 0.f;
+        uint32_t msk = 0;
+        // the accepted centres 16 at a time: one TMEM column each
+        for (int j0 = 0; j0 < nA; j0 += 16) {
+          uint32_t dv_[16];
 #pragma unroll
-          for (int j = 0; j < kMaxAccept; ++j) {
-            if (j < nA) {
-              const float d = __fsub_rn(1.0f, __fmul_rn(__fmul_rn(__uint_as_float(dv_[j]), ri), rc[j]));
-              if (!(__fsub_rn(d, eps) >= dl)) msk |= 1u << j;   // NaN also goes to the exact path
+          for (int j = 0; j < 16; ++j)
+            if (j0 + j < nA) tmem_ld1(tbase + (uint32_t)lp_row[acc_s[j0 + j]], &dv_[j]);
+          tmem_wait_ld();
+#pragma unroll
+          for (int j = 0; j < 16; ++j) {
+            if (j0 + j < nA) {
+              const float rcj = lp_f[acc_s[j0 + j] * 3 + 2];
+              const float d = __fsub_rn(1.0f, __fmul_rn(__fmul_rn(__uint_as_float(dv_[j]), ri), rcj));
+              if (!(__fsub_rn(d, eps) >= dl)) msk |= 1u << (j0 + j);   // NaN also goes to the exact path
             }
           }
-          if (msk) {
-            const int pos = atomicAdd(fcnt, 1);
-            fidx[pos] = t;
-            fmask[pos] = (unsigned short)msk;
-          }
+        }
+        if (live && msk) {
+          const int pos = atomicAdd(fcnt, 1);
+          fidx[pos] = t;
+          fmask[pos] = msk;
         }
       }
       tc_fence_before();
@@ -758,7 +760,7 @@ select_kernel(const __grid_constant__ SelectArgs a) {
       }
       __syncthreads();
       // 5. keys of the unselected tokens -> the warp's ranked list for the next round
-      TopList tl;
+      TopList<kTop> tl;
       tl.clear();
       for (int t0 = warp * 32; t0 < nloc; t0 += kSelectWarps * 32) {
         const int t = t0 + lane;
@@ -766,18 +768,18 @@ select_kernel(const __grid_constant__ SelectArgs a) {
             (t < nloc && !sel_s[t]) ? argmax_key(__fmul_rn(w_s[t], dl_s[t]), lo + t) : 0ull;
         // the warp's 32 keys enter the list in descending order
         unsigned long long kk = key;
-        for (int i = 0; i < kTopM; ++i) {
+        for (int i = 0; i < kTop; ++i) {
           const uint32_t hi = __reduce_max_sync(0xffffffffu, (uint32_t)(kk >> 32));
           const uint32_t lo_ = __reduce_max_sync(0xffffffffu, (uint32_t)(kk >> 32) == hi ? (uint32_t)kk : 0u);
           const unsigned long long best = ((unsigned long long)hi << 32) | lo_;
-          if (best == 0ull || best <= tl.k[kTopM - 1]) break;
+          if (best == 0ull || best <= tl.k[kTop - 1]) break;
           tl.insert(best);
           if (kk == best) kk = 0ull;
         }
       }
       if (lane == 0) {
 #pragma unroll
-        for (int i = 0; i < kTopM; ++i) wtop[warp * kTopM + i] = tl.k[i];
+        for (int i = 0; i < kTop; ++i) wtop[warp * kTop + i] = tl.k[i];
       }
     };
     auto update = [&](int nA) {
@@ -798,10 +800,10 @@ select_kernel(const __grid_constant__ SelectArgs a) {
       unsigned long long best = 0ull;
       int bq = 0;
       for (int q = 0; q < C; ++q) {
-        const unsigned long long kq = pub_key[(0 * kMaxCluster + q) * kTopM];
+        const unsigned long long kq = pub_key[(0 * kMaxCluster + q) * kTopMax];
         if (kq > best) { best = kq; bq = q; }
       }
-      const int slot = (0 * kMaxCluster + bq) * kTopM;
+      const int slot = (0 * kMaxCluster + bq) * kTopMax;
       lp_key[0] = best;
       lp_idx[0] = key_index(best);
       const float4 f = pub_f[slot];
@@ -830,7 +832,7 @@ select_kernel(const __grid_constant__ SelectArgs a) {
       if (TC && early && warp > 0) {   // warps 1.. copy while warp 0 builds the list
         for (int q = 0; q < C; ++q)
           for (int e = 0; e < a.mc; ++e) {
-            const unsigned long long kq = pub_key[(par * kMaxCluster + q) * kTopM + e];
+            const unsigned long long kq = pub_key[(par * kMaxCluster + q) * kTopMax + e];
             if (kq != 0ull) copy_row_tc(q * a.mc + e, key_index(kq), 32, kSelThreads - 32);
           }
         cp_async_commit();
@@ -838,11 +840,11 @@ select_kernel(const __grid_constant__ SelectArgs a) {
         uint32_t bytes = 0;
         for (int q = 0; q < C; ++q)
           for (int e = 0; e < a.mc; ++e)
-            bytes += pub_key[(par * kMaxCluster + q) * kTopM + e] != 0ull ? (uint32_t)rb : 0u;
+            bytes += pub_key[(par * kMaxCluster + q) * kTopMax + e] != 0ull ? (uint32_t)rb : 0u;
         mbar_expect_tx(bar, bytes);
         for (int q = 0; q < C; ++q)
           for (int e = 0; e < a.mc; ++e) {
-            const unsigned long long kq = pub_key[(par * kMaxCluster + q) * kTopM + e];
+            const unsigned long long kq = pub_key[(par * kMaxCluster + q) * kTopMax + e];
             if (kq != 0ull)
               bulk_g2s(cbuf + (long long)(q * a.mc + e) * rb, xreq + (long long)key_index(kq) * rb,
                        (uint32_t)rb, bar);
@@ -852,18 +854,18 @@ select_kernel(const __grid_constant__ SelectArgs a) {
       if (warp == 0) {
         const int kPer = a.mc;
         const int ne = C * kPer;
-        const unsigned long long u5 = lane < C ? pub_key[(par * kMaxCluster + lane) * kTopM + kPer] : 0ull;
+        const unsigned long long u5 = lane < C ? pub_key[(par * kMaxCluster + lane) * kTopMax + kPer] : 0ull;
         const uint32_t uhi = __reduce_max_sync(0xffffffffu, (uint32_t)(u5 >> 32));
         const uint32_t ulo = __reduce_max_sync(0xffffffffu, (uint32_t)(u5 >> 32) == uhi ? (uint32_t)u5 : 0u);
         const unsigned long long U = ((unsigned long long)uhi << 32) | ulo;
         int slot0 = 0, slot1 = 0;
         unsigned long long ke0 = 0ull, ke1 = 0ull;
         if (lane < ne) {
-          slot0 = (par * kMaxCluster + lane / kPer) * kTopM + lane % kPer;
+          slot0 = (par * kMaxCluster + lane / kPer) * kTopMax + lane % kPer;
           ke0 = pub_key[slot0];
         }
         if (lane + 32 < ne) {
-          slot1 = (par * kMaxCluster + (lane + 32) / kPer) * kTopM + (lane + 32) % kPer;
+          slot1 = (par * kMaxCluster + (lane + 32) / kPer) * kTopMax + (lane + 32) % kPer;
           ke1 = pub_key[slot1];
         }
         const bool c0 = ke0 > U, c1 = ke1 > U;
@@ -883,7 +885,7 @@ select_kernel(const __grid_constant__ SelectArgs a) {
             const float4 f = pub_f[slot];
             lp_key[pos] = ke;
             lp_idx[pos] = key_index(ke);
-            lp_row[pos] = (slot % kTopM) + (slot / kTopM - par * kMaxCluster) * a.mc;
+            lp_row[pos] = (slot % kTopMax) + (slot / kTopMax - par * kMaxCluster) * a.mc;
             lp_f[pos * 3 + 0] = f.x;
             lp_f[pos * 3 + 1] = f.y;
             lp_f[pos * 3 + 2] = f.z;
@@ -930,16 +932,22 @@ select_kernel(const __grid_constant__ SelectArgs a) {
             if (col < dv) {
 #pragma unroll
               for (int j = 0; j < 4; ++j) {
-                float ea[8], eb[8];
                 if constexpr (TC) {
-                  Elem<T>::widen(lds32(cb_chunk(ja[j], col)), ea);
-                  Elem<T>::widen(lds32(cb_chunk(jv[j], col)), eb);
+                  // bf16 rows: one mixed-precision fma per coordinate, in the same order
+                  const U4 va = lds32(cb_chunk(ja[j], col)), vb = lds32(cb_chunk(jv[j], col));
+                  const uint32_t wa[4] = {va.x, va.y, va.z, va.w}, wb[4] = {vb.x, vb.y, vb.z, vb.w};
+#pragma unroll
+                  for (int hw = 0; hw < 4; ++hw) {
+                    acc[j] = fma_bf16_lo(wa[hw], wb[hw], acc[j]);
+                    acc[j] = fma_bf16_hi(wa[hw], wb[hw], acc[j]);
+                  }
                 } else {
+                  float ea[8], eb[8];
                   load8<T, true>(cbuf + (long long)ja[j] * rb, col, ea);
                   load8<T, true>(cbuf + (long long)jv[j] * rb, col, eb);
-                }
 #pragma unroll
-                for (int q = 0; q < 8; ++q) acc[j] = __fmaf_rn(ea[q], eb[q], acc[j]);
+                  for (int q = 0; q < 8; ++q) acc[j] = __fmaf_rn(ea[q], eb[q], acc[j]);
+                }
               }
             }
           }
@@ -962,7 +970,7 @@ select_kernel(const __grid_constant__ SelectArgs a) {
         const float rv = pending ? lp_f[lane * 3 + 2] : 0.f;
         const int gi = pending ? lp_idx[lane] : 0;
         int nA = 0;
-        while (taken + nA < K && nA < kMaxAccept) {
+        while (taken + nA < K && nA < a.max_accept) {
           // argmax of the pending keys: high word (ordered value) then low word (index)
           const uint32_t khi = pending ? (uint32_t)(key >> 32) : 0u;
           const uint32_t mhi = __reduce_max_sync(0xffffffffu, khi);

@@ -219,13 +219,14 @@ cudaError_t launch_select(const Plan &pl, const float *w, const void *x, int32_t
     double round_cycles;
     if (tc) {
       // The update streams this CTA's rows (whole 128-row tiles) once per round, at
-      // the smaller of the ring's hand-off rate (about 900 cycles per stage, measured)
-      // and this CTA's share of DRAM (or of L2, taken as 2.5x, when the features of
-      // the requests in flight fit in it).
+      // the smallest of the ring's hand-off rate (about 900 cycles per stage), the
+      // rate one SM's TMA sustains (about 26 bytes per clock; both measured on
+      // GB300) and this CTA's share of DRAM (or of L2, taken as 2.5x, when the
+      // features of the requests in flight fit in it).
       const double bytes = (double)((tpc_c + kTcBM - 1) / kTcBM) * kTcBM * tc_kblocks(pl.dv) * 128.0;
       const double ctas = std::min<double>(pl.B, active) * c;
       const double share = di.dram_bytes_per_cycle / ctas * (from_hbm ? 1.0 : 2.5);
-      const double bw = std::min(kps_c * (double)kTcBoxBytes / 900.0, share);
+      const double bw = std::min(std::min(kps_c * (double)kTcBoxBytes / 900.0, 26.0), share);
       round_cycles = bytes / bw + 30000.0 + 400.0 * c;
     } else {
       const double stream_penalty = from_hbm ? 3.0 : 1.0;
@@ -248,8 +249,17 @@ cudaError_t launch_select(const Plan &pl, const float *w, const void *x, int32_t
   a.meta = reinterpret_cast<const int32_t *>(ws + pl.off_meta);
   a.order = reinterpret_cast<const int32_t *>(ws + pl.off_order);
   a.dv = pl.dv; a.row_bytes = rb; a.tpc_max = tpc; a.cache_rows = cache_rows; a.csize = C;
-  // enough candidates per CTA that the list approximates the global top 16
-  a.mc = C <= 4 ? kTopM - 1 : 4;
+  // Candidates each CTA publishes: enough that the list approximates the global
+  // top picks, at most 64 in all (the list is built by one warp, two per lane).
+  // The tensor-core update ranks 16 per CTA and accepts up to 32 picks a round;
+  // the CUDA-core update ranks 8 and accepts 16 (its register blocking).
+  if (tc) {
+    a.mc = std::min(16, 64 / C);
+    a.max_accept = kMaxAccept;
+  } else {
+    a.mc = C <= 4 ? 8 : 4;
+    a.max_accept = 16;
+  }
   a.ring = ring;
   a.lcap = lcap;
   a.err = reinterpret_cast<unsigned *>(ws + pl.off_err);
