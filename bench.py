@@ -369,7 +369,7 @@ def main():
     select_ms = statistics.mean(e[1].elapsed_time(e[2]) for e in ev)
     total_ms, reqs, toks = combine_over_ranks(total_ms, wl.batch * K, nvis * K, device=dev)
     value = reqs / (total_ms / 1e3)
-    tokens_per_s = toks / (total_ms / 1e3)
+    tokens_per_s = toks / (scores_ms * K / 1e3)   # visual tokens scored per second of scoring
 
     pk, pk_kind = peaks()
     hbm = float(pk.get("hbm_gbs", FALLBACK_HBM_GBS))
