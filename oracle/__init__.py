@@ -77,6 +77,9 @@ def _load():
         lib.oracle_select_fp32.restype = i32
         lib.oracle_select_fp64.argtypes = [i32, i32, i32, P, P, i32, P]
         lib.oracle_select_fp64.restype = i32
+        lib.oracle_scores_rows.argtypes = [i32, i32, i32, i32, i32, i32, ctypes.c_double,
+                                           P, P, P, P, P, P, P, P]
+        lib.oracle_scores_rows.restype = i32
         lib.oracle_select_topk.argtypes = [i32, P, i32, P]
         lib.oracle_select_topk.restype = i32
         lib.oracle_restore_order.argtypes = [i32, P, P]
@@ -132,6 +135,27 @@ def scores(q, k, cu_seqlens, vis_start, cu_vis, *, num_kv_heads, scale=0.0):
                                _ptr(cu), _ptr(vs), _ptr(cv), _ptr(q), _ptr(k), _ptr(out))
     if rc:
         raise ValueError(f"oracle_scores rejected its arguments (rc={rc})")
+    return out
+
+
+def scores_rows(q_rows, k, cu_seqlens, vis_start, cu_vis, cu_rows, row_pos, *, num_kv_heads,
+                scale=0.0):
+    """Table 4's attention sources in fp64: q_rows [sum M][L][Hq][D] holds the query
+    rows of every request (cu_rows offsets, request-local positions row_pos); returns
+    w [sum N] float64."""
+    R, L, Hq, D = q_rows.shape
+    assert k.ndim == 4 and k.shape[0] == L and k.shape[2] == num_kv_heads and k.shape[3] == D
+    assert q_rows.dtype == k.dtype
+    cu, vs, cv = _i32(cu_seqlens), _i32(vis_start), _i32(cu_vis)
+    cr, rp = _i32(cu_rows), _i32(row_pos)
+    B = len(cu) - 1
+    assert int(cr[-1]) == R and len(rp) == R
+    out = np.zeros(int(cv[-1]), dtype=np.float64)
+    rc = _load().oracle_scores_rows(B, L, Hq, num_kv_heads, D, _dtype_code(q_rows), float(scale),
+                                    _ptr(cu), _ptr(vs), _ptr(cv), _ptr(cr), _ptr(rp),
+                                    _ptr(np.ascontiguousarray(q_rows)), _ptr(k), _ptr(out))
+    if rc:
+        raise ValueError(f"oracle_scores_rows rejected its arguments (rc={rc})")
     return out
 
 

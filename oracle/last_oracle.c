@@ -12,6 +12,8 @@
  * paper states them:
  *   oracle_last_row        Eq. 6  (one row p* of the causal softmax attention)
  *   oracle_scores          Eq. 6, 7, 8 (sum over layers and heads, normalise)
+ *   oracle_scores_rows     Table 4's attention sources: Eq. 6-8 with the rows of
+ *                          several query positions summed (First, Middle, All Mean)
  *   oracle_select_fp32     Eq. 9, 10, 11 in "canonical fp32" arithmetic
  *   oracle_select_fp64     Eq. 9, 10, 11 in plain fp64 arithmetic
  *   oracle_select_topk     Table 5's "Top-k" selection: the k highest scores
@@ -295,6 +297,74 @@ int oracle_select_topk(int N, const float *w, int k, int32_t *order_out) {
     taken[best] = 1;
   }
   free(taken);
+  return 0;
+}
+
+/* Table 4 (attention sources): the importance of Eq. 7 taken from the attention
+ * rows of several query positions instead of p* alone.  Request b has the query
+ * rows cu_rows[b] .. cu_rows[b+1]-1; row r sits at request-local position
+ * row_pos[r], after the visual span (vis_start[b] + N_b <= row_pos[r] <= P_b - 1),
+ * and its causal softmax runs over the keys 0 .. row_pos[r].  q holds one query
+ * vector per row, layer and q-head: [cu_rows[B]][L][Hq][D].  The rows' probabilities
+ * at the visual positions are summed over rows, layers and heads (a mean over the
+ * rows is the same after Eq. 8's normalisation), then normalised. */
+int oracle_scores_rows(int B, int L, int Hq, int Hkv, int D, int dtype, double scale,
+                       const int32_t *cu_seqlens, const int32_t *vis_start, const int32_t *cu_vis,
+                       const int32_t *cu_rows, const int32_t *row_pos, const void *q,
+                       const void *k, double *w_out) {
+  if (Hkv <= 0 || Hq % Hkv != 0 || cu_rows[0] != 0) return 1;
+  if (scale <= 0.0) scale = 1.0 / sqrt((double)D);
+  const int group = Hq / Hkv;
+  const int64_t total_keys = cu_seqlens[B];
+  int max_p = 1;
+  for (int b = 0; b < B; ++b) {
+    const int P = cu_seqlens[b + 1] - cu_seqlens[b];
+    const int N = cu_vis[b + 1] - cu_vis[b];
+    if (P <= 0 || N < 0 || vis_start[b] < 0) return 1;
+    if (cu_rows[b + 1] <= cu_rows[b]) return 1;          /* at least one row */
+    for (int r = cu_rows[b]; r < cu_rows[b + 1]; ++r)
+      if (row_pos[r] < vis_start[b] + N || row_pos[r] > P - 1) return 1;
+    if (P > max_p) max_p = P;
+  }
+  double *a = (double *)malloc(sizeof(double) * (size_t)max_p);
+  if (!a) return 2;
+  for (int b = 0; b < B; ++b) {
+    const int N = cu_vis[b + 1] - cu_vis[b];
+    const int64_t p0 = cu_seqlens[b];
+    double *s = w_out + cu_vis[b];
+    for (int i = 0; i < N; ++i) s[i] = 0.0;
+    for (int r = cu_rows[b]; r < cu_rows[b + 1]; ++r) {
+      const int pos = row_pos[r];
+      for (int l = 0; l < L; ++l) {
+        for (int h = 0; h < Hq; ++h) {
+          const int g = h / group;
+          const int64_t qoff = (((int64_t)r * L + l) * Hq + h) * D;
+          /* Eq. 6 for this row: causal softmax over keys 0..pos */
+          double zmax = -INFINITY;
+          for (int p = 0; p <= pos; ++p) {
+            const int64_t koff = (((int64_t)l * total_keys + p0 + p) * Hkv + g) * D;
+            double acc = 0.0;
+            for (int d = 0; d < D; ++d)
+              acc += load_elem(q, dtype, qoff + d) * load_elem(k, dtype, koff + d);
+            a[p] = scale * acc;
+            if (a[p] > zmax) zmax = a[p];
+          }
+          double zsum = 0.0;
+          for (int p = 0; p <= pos; ++p) {
+            a[p] = exp(a[p] - zmax);
+            zsum += a[p];
+          }
+          /* Eq. 7: accumulate the visual positions */
+          for (int i = 0; i < N; ++i) s[i] += a[vis_start[b] + i] / zsum;
+        }
+      }
+    }
+    /* Eq. 8 */
+    double total = 0.0;
+    for (int i = 0; i < N; ++i) total += s[i];
+    for (int i = 0; i < N; ++i) s[i] = s[i] / total;
+  }
+  free(a);
   return 0;
 }
 

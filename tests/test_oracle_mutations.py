@@ -16,11 +16,15 @@ SRC = os.path.join(ROOT, "oracle", "last_oracle.c")
 
 # (name, exact substring in the source, replacement)
 MUTANTS = [
-    ("gqa_mapping_modulo", "const int g = h / group;", "const int g = h % Hkv;"),
+    ("gqa_mapping_modulo", "const int g = h / group;\n  const int64_t total_keys",
+     "const int g = h % Hkv;\n  const int64_t total_keys"),
     ("query_key_dropped", "for (int p = 0; p < P; ++p) {\n    const int64_t koff",
      "for (int p = 0; p < P - 1; ++p) {\n    const int64_t koff"),
     ("scale_dropped", "a_out[p] = scale * acc;", "a_out[p] = acc;"),
-    ("no_visual_normalisation", "s[i] = s[i] / total;", "s[i] = s[i] / (double)(L * Hq);"),
+    ("no_visual_normalisation", "s[i] = s[i] / total;\n  }\n  free(row);",
+     "s[i] = s[i] / (double)(L * Hq);\n  }\n  free(row);"),
+    ("rows_no_visual_normalisation", "s[i] = s[i] / total;\n  }\n  free(a);",
+     "s[i] = s[i] / (double)(L * Hq);\n  }\n  free(a);"),
     ("visual_offset_ignored", "s[i] += row[vis_start[b] + i];", "s[i] += row[i];"),
     ("distance_sign", "float dist = 1.0f - c;", "float dist = 1.0f + c;"),
     ("wrong_norm_index", "float c = (dot * r[i]) * r[j];", "float c = (dot * r[i]) * r[i];"),
@@ -37,11 +41,18 @@ MUTANTS = [
      "if (best < 0 || w[i] >= w[best]) best = i;"),
     ("topk_lowest_scores", "if (best < 0 || w[i] > w[best]) best = i;",
      "if (best < 0 || w[i] < w[best]) best = i;"),
+    ("rows_causal_extent_short", "for (int p = 0; p <= pos; ++p) {\n            const int64_t koff",
+     "for (int p = 0; p < pos; ++p) {\n            const int64_t koff"),
+    ("rows_position_ignored", "const int pos = row_pos[r];",
+     "const int pos = cu_seqlens[b + 1] - cu_seqlens[b] - 1;"),
+    ("rows_gqa_modulo", "const int g = h / group;\n          const int64_t qoff = (((int64_t)r",
+     "const int g = h % Hkv;\n          const int64_t qoff = (((int64_t)r"),
 ]
 
 PIN_FILES = [os.path.join(ROOT, "tests", "test_oracle_scores.py"),
              os.path.join(ROOT, "tests", "test_oracle_select.py"),
-             os.path.join(ROOT, "tests", "test_oracle_topk.py")]
+             os.path.join(ROOT, "tests", "test_oracle_topk.py"),
+             os.path.join(ROOT, "tests", "test_oracle_rows.py")]
 
 
 def _run_pins(lib):
