@@ -124,6 +124,25 @@ last_status last_select_topk(const last_problem *p, const float *w, const void *
                              int32_t *idx_out, void *x_out, void *ws, size_t ws_bytes,
                              void *stream);
 
+/* Table 4 (attention sources: First, Middle, All Mean): Eq. 6-8 with the
+ * attention rows of several query positions per request instead of p* alone.
+ * Request b's query rows are cu_rows[b] .. cu_rows[b+1]-1 (HOST array, length
+ * batch+1, cu_rows[0] = 0, at least one row per request); row r sits at the
+ * request-local position row_pos[r] (HOST array), which must lie after the visual
+ * span: vis_start[b] + N_b <= row_pos[r] <= P_b - 1; row r's softmax runs over the
+ * keys 0 .. row_pos[r] (causal).  q_rows [cu_rows[batch]][num_layers][num_q_heads]
+ * [head_dim] holds one query vector per row, layer and q-head; k as for
+ * last_scores.  w_out [cu_vis[batch]] receives the visual probabilities summed
+ * over rows, layers and q-heads and normalised per request (a mean over the rows
+ * gives the same w~).  Limits: bf16 only; head_dim 64, 128, 192 or 256; rows x
+ * (num_q_heads / num_kv_heads) <= 256 and rows x layers x q-heads <= 6144 per
+ * request.  The workspace is sized by last_scores_rows_workspace_size. */
+last_status last_scores_rows_workspace_size(const last_problem *p, const int32_t *cu_rows,
+                                            const int32_t *row_pos, size_t *bytes);
+last_status last_scores_rows(const last_problem *p, const int32_t *cu_rows,
+                             const int32_t *row_pos, const void *q_rows, const void *k,
+                             float *w_out, void *ws, size_t ws_bytes, void *stream);
+
 /* Eq. 12.  x_out[r] = x[cu_vis[b] + idx[r]] for r in request b's output range.
  * An index outside [0, N_b) leaves its row unwritten and makes last_poll
  * return LAST_ERR_DEVICE_INDEX. */

@@ -34,7 +34,8 @@ LAST_DTYPE_BF16 = 1
 
 EXPORTED = ("last_workspace_size", "last_scores", "last_select", "last_gather", "last_prune",
             "last_poll", "last_budget", "last_status_string", "last_error_message",
-            "last_scores_noalloc", "last_select_topk")
+            "last_scores_noalloc", "last_select_topk", "last_scores_rows",
+            "last_scores_rows_workspace_size")
 
 
 class LastError(RuntimeError):
@@ -77,6 +78,9 @@ def load_library(path: str = LIB_PATH):
     lib.last_select.argtypes = [PP, P, P, P, P, P, ctypes.c_size_t, P]
     lib.last_gather.argtypes = [PP, P, P, P, P, ctypes.c_size_t, P]
     lib.last_select_topk.argtypes = [PP, P, P, P, P, P, ctypes.c_size_t, P]
+    PI = ctypes.POINTER(ctypes.c_int32)
+    lib.last_scores_rows.argtypes = [PP, PI, PI, P, P, P, P, ctypes.c_size_t, P]
+    lib.last_scores_rows_workspace_size.argtypes = [PP, PI, PI, ctypes.POINTER(ctypes.c_size_t)]
     lib.last_prune.argtypes = [PP, P, P, P, P, P, P, P, ctypes.c_size_t, P]
     lib.last_poll.argtypes = [P, P]
     lib.last_scores_noalloc.argtypes = [PP, P, P, P, P]
@@ -87,7 +91,8 @@ def load_library(path: str = LIB_PATH):
     lib.last_error_message.argtypes = []
     lib.last_error_message.restype = ctypes.c_char_p
     for name in ("last_workspace_size", "last_scores", "last_select", "last_gather",
-                 "last_prune", "last_poll", "last_scores_noalloc", "last_select_topk"):
+                 "last_prune", "last_poll", "last_scores_noalloc", "last_select_topk",
+                 "last_scores_rows", "last_scores_rows_workspace_size"):
         getattr(lib, name).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -196,6 +201,37 @@ def last_select_topk(problem: Problem, w, idx_out, ws, stream=None, x=None, x_ou
     p, n = _ws(ws)
     _check(load_library().last_select_topk(problem.ref, _ptr(w), _ptr(x), _ptr(idx_out),
                                            _ptr(x_out), p, n, _stream(stream)))
+
+
+class QueryRows:
+    """Query rows of Table 4's attention sources: per-request offsets cu_rows
+    [batch + 1] and request-local positions row_pos (host int32 arrays)."""
+
+    def __init__(self, cu_rows: Sequence[int], row_pos: Sequence[int]):
+        self.cu_rows = np.ascontiguousarray(np.asarray(cu_rows, dtype=np.int32))
+        self.row_pos = np.ascontiguousarray(np.asarray(row_pos, dtype=np.int32))
+        I = ctypes.POINTER(ctypes.c_int32)
+        self.c_cu = self.cu_rows.ctypes.data_as(I)
+        self.c_pos = self.row_pos.ctypes.data_as(I)
+
+
+def last_scores_rows_workspace_size(problem: Problem, rows: QueryRows) -> int:
+    n = ctypes.c_size_t(0)
+    _check(load_library().last_scores_rows_workspace_size(problem.ref, rows.c_cu, rows.c_pos,
+                                                          ctypes.byref(n)))
+    return n.value
+
+
+def rows_workspace(problem: Problem, rows: QueryRows, device="cuda"):
+    import torch
+    return torch.empty(max(last_scores_rows_workspace_size(problem, rows), 256), dtype=torch.uint8,
+                       device=device)
+
+
+def last_scores_rows(problem: Problem, rows: QueryRows, q_rows, k, w_out, ws, stream=None):
+    p, n = _ws(ws)
+    _check(load_library().last_scores_rows(problem.ref, rows.c_cu, rows.c_pos, _ptr(q_rows),
+                                           _ptr(k), _ptr(w_out), p, n, _stream(stream)))
 
 
 def last_gather(problem: Problem, x, idx, x_out, ws, stream=None):

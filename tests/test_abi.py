@@ -104,6 +104,30 @@ def test_topk_needs_no_sequence_fields(lib):
     assert e.value.status == last.LAST_ERR_WORKSPACE_TOO_SMALL
 
 
+@pytest.mark.parametrize("kw,rows,status", [
+    (dict(dtype="f32"), ([0, 1, 2], [8, 20]), last.LAST_ERR_UNSUPPORTED),          # bf16 only
+    (dict(), ([0, 1, 2], [5, 20]), last.LAST_ERR_INVALID_ARG),                     # inside span
+    (dict(), ([0, 1, 2], [8, 20]), last.LAST_ERR_INVALID_ARG),                     # past P_b - 1
+    (dict(), ([0, 0, 2], [20, 21]), last.LAST_ERR_INVALID_ARG),                    # no row
+    (dict(head_dim=80), ([0, 1, 2], [8, 20]), last.LAST_ERR_UNSUPPORTED),          # head_dim
+    (dict(num_q_heads=16, num_kv_heads=2), ([0, 33, 34], list(range(6, 10)) * 8 + [9, 19]),
+     last.LAST_ERR_UNSUPPORTED),                                                 # 33 x 8 > 256
+])
+def test_scores_rows_rejects_bad_arguments(lib, kw, rows, status):
+    prob = _problem(**kw)
+    qr = last.QueryRows(*rows)
+    with pytest.raises(last.LastError) as e:
+        last.last_scores_rows(prob, qr, 16, 16, 16, (256, 1 << 30), stream=0)
+    assert e.value.status == status
+
+
+def test_scores_rows_workspace_grows_with_rows(lib):
+    prob = _problem()
+    one = last.last_scores_rows_workspace_size(prob, last.QueryRows([0, 1, 2], [9, 19]))
+    many = last.last_scores_rows_workspace_size(prob, last.QueryRows([0, 3, 6], [6, 7, 9, 10, 15, 19]))
+    assert many > one > 0
+
+
 def test_workspace_checks(lib):
     prob = _problem()
     need = last.last_workspace_size(prob)
