@@ -48,6 +48,11 @@ def parse():
     ap.add_argument("--selector", default="greedy", choices=["greedy", "topk"],
                     help="greedy: importance-weighted k-center (Eq. 9-11, the method); "
                          "topk: the Top-k variant of Table 5")
+    ap.add_argument("--source", default="last", choices=["last", "first", "middle", "all"],
+                    help="attention source of the importance scores (Table 4): the last query "
+                         "row (the method), the first or middle text row, or the mean of up "
+                         "to --rows text rows")
+    ap.add_argument("--rows", type=int, default=32, help="rows per request for --source all")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     return ap.parse_args()
@@ -222,14 +227,24 @@ def peaks():
         return {"hbm_gbs": FALLBACK_HBM_GBS, "sm_max_mhz": 2070.0}, "fallback"
 
 
-def oracle_request(oracle, wl, b, selector="greedy"):
-    """One whole request through the oracle: fp64 scores of the request, then the
-    canonical-fp32 greedy (or Top-k), order restore and gather.  Returns N_b."""
+def oracle_request(oracle, wl, b, selector="greedy", rows=None):
+    """One whole request through the oracle: fp64 scores of the request (from its
+    last query row, or from the query rows `rows` = (cu_rows, row_pos, q_rows) of
+    another attention source), then the canonical-fp32 greedy (or Top-k), order
+    restore and gather.  Returns N_b."""
     v0, v1 = int(wl.cu_vis[b]), int(wl.cu_vis[b + 1])
     s0, s1 = int(wl.cu_seqlens[b]), int(wl.cu_seqlens[b + 1])
     kb = int(wl.cu_keep[b + 1] - wl.cu_keep[b])
-    w = oracle.scores(wl.q[b:b + 1], np.ascontiguousarray(wl.k[:, s0:s1]), [0, s1 - s0],
-                      [int(wl.vis_start[b])], [0, v1 - v0], num_kv_heads=wl.num_kv_heads)
+    kreq = np.ascontiguousarray(wl.k[:, s0:s1])
+    if rows is None:
+        w = oracle.scores(wl.q[b:b + 1], kreq, [0, s1 - s0], [int(wl.vis_start[b])], [0, v1 - v0],
+                          num_kv_heads=wl.num_kv_heads)
+    else:
+        cu, pos, qr = rows
+        r0, r1 = int(cu[b]), int(cu[b + 1])
+        w = oracle.scores_rows(np.ascontiguousarray(qr[r0:r1]), kreq, [0, s1 - s0],
+                               [int(wl.vis_start[b])], [0, v1 - v0], [0, r1 - r0], pos[r0:r1],
+                               num_kv_heads=wl.num_kv_heads)
     w32 = w.astype(np.float32)
     if selector == "topk":
         oracle.gather(wl.x[v0:v1], oracle.restore_order(oracle.select_topk(w32, kb)))
@@ -238,7 +253,7 @@ def oracle_request(oracle, wl, b, selector="greedy"):
     return v1 - v0
 
 
-def cpu_baseline(wl, budget_s=15.0, selector="greedy"):
+def cpu_baseline(wl, budget_s=15.0, selector="greedy", rows=None):
     """The oracle as it stands (single thread) on a bounded sample of the same batch:
     whole requests in batch order until about budget_s seconds have passed."""
     import oracle
@@ -246,7 +261,7 @@ def cpu_baseline(wl, budget_s=15.0, selector="greedy"):
     t0 = time.perf_counter()
     done = 0
     for b in range(wl.batch):
-        oracle_request(oracle, wl, b, selector)
+        oracle_request(oracle, wl, b, selector, rows)
         done += 1
         if time.perf_counter() - t0 > budget_s:
             break
@@ -261,12 +276,16 @@ def run_reference(args, rank, world):
     if rank != 0:
         return
     wl = workload(args.budget, 0, args.workload)
+    rows = None
+    if args.source != "last":
+        from workloads import query_rows
+        rows = query_rows(wl, args.source, args.rows)
     import oracle
     oracle.build()
 
     def step(i):
         # a bounded sample per step: one whole request of the batch, in turn
-        return oracle_request(oracle, wl, i % wl.batch, args.selector)
+        return oracle_request(oracle, wl, i % wl.batch, args.selector, rows)
 
     for i in range(args.warmup):
         step(i)
@@ -281,7 +300,8 @@ def run_reference(args, rank, world):
             "ms_per_step": 1000 * dt / args.steps, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64 scores / f32 selection", "data": "synthetic",
             "config": workload_desc(wl, args.budget, args.workload)
-                      | {"per_step": "1 whole request (oracle)", "selector": args.selector},
+                      | {"per_step": "1 whole request (oracle)", "selector": args.selector,
+                         "source": args.source},
             "visual_tokens_scored_per_s": toks / dt,
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
                              "sample": f"1 whole request of the {args.workload} batch per step, "
@@ -330,6 +350,19 @@ def main():
     stream = torch.cuda.current_stream(dev)
 
     topk = args.selector == "topk"
+    rows = rows_host = None
+    if args.source != "last":
+        from workloads import query_rows
+        rows_host = query_rows(wl, args.source, args.rows)
+        rows = last.QueryRows(rows_host[0], rows_host[1])
+        q_rows = dev_t(rows_host[2])
+        ws_rows = last.rows_workspace(prob, rows, dev)
+
+    def score():
+        if rows is None:
+            last.last_scores(prob, q, k, w, ws, stream)
+        else:
+            last.last_scores_rows(prob, rows, q_rows, k, w, ws_rows, stream)
 
     def select():
         if topk:
@@ -338,7 +371,7 @@ def main():
             last.last_select(prob, w, x, idx, ws, stream, x_out=xs)
 
     def step():
-        last.last_scores(prob, q, k, w, ws, stream)
+        score()
         select()
 
     for _ in range(args.warmup):
@@ -356,7 +389,7 @@ def main():
         torch.cuda.synchronize(dev)
         for i in range(K):
             ev[i][0].record(stream)
-            last.last_scores(prob, q, k, w, ws, stream)
+            score()
             ev[i][1].record(stream)
             select()
             ev[i][2].record(stream)
@@ -373,11 +406,14 @@ def main():
 
     pk, pk_kind = peaks()
     hbm = float(pk.get("hbm_gbs", FALLBACK_HBM_GBS))
-    sc_gbs = score_bytes(wl) / (scores_ms / 1e3) / 1e9
+    sc_bytes = score_bytes(wl) if rows is None else (
+        wl.k.nbytes + rows_host[2].nbytes + 4 * int(wl.cu_vis[-1]))
+    sc_gbs = sc_bytes / (scores_ms / 1e3) / 1e9
 
     e2e = None
     if not args.no_e2e:
-        e2e = measure_e2e(args, wl, prob, dev, stream, last, q, k, x)
+        e2e = measure_e2e(args, wl, prob, dev, stream, last, q, k, x,
+                          None if rows is None else (rows, rows_host[2], q_rows, ws_rows))
 
     comp, greedy = prune_bytes_moved(wl)
     sel_gbs = greedy / (select_ms / 1e3) / 1e9
@@ -421,17 +457,27 @@ def main():
                             "peak_note": f"{pk_kind} HBM copy bandwidth; achieved = compulsory "
                                          "scoring bytes / event time of last_scores"}
         line["kernels"]["topk_gather_ms"] = line["kernels"].pop("select_ms")
+    if rows is not None:
+        # Table 4's attention source: the logits are a bf16 tensor-core contraction of
+        # every key with the request's query rows
+        cu = rows_host[0]
+        flops = 2.0 * sum(int(wl.cu_seqlens[b + 1] - wl.cu_seqlens[b]) * int(cu[b + 1] - cu[b])
+                          for b in range(wl.batch)) * wl.num_q_heads * wl.head_dim * wl.num_layers
+        line["config"]["source"] = f"{args.source} ({int(cu[-1])} query rows, Table 4)"
+        line["kernels"]["scores_tensor_TFLOPs"] = flops / (scores_ms / 1e3) / 1e12
+        if topk:
+            line["roofline"]["kernel"] = "rows_logits_kernel+rows_tokens_kernel"
     if e2e is not None:
         line["e2e"] = e2e
     if rank == 0 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(wl, selector=args.selector)
+        line["cpu_baseline"] = cpu_baseline(wl, selector=args.selector, rows=rows_host)
     if rank == 0:
         print(json.dumps(line), flush=True)
     if world > 1:
         torch.distributed.destroy_process_group()
 
 
-def measure_e2e(args, wl, prob, dev, stream, last, q_d, k_d, x_d):
+def measure_e2e(args, wl, prob, dev, stream, last, q_d, k_d, x_d, rows=None):
     """The same metric through the user call last_prune with host buffers: each step
     copies q, K, X from pinned host memory, prunes, and reads back the kept indices and
     rows."""
@@ -440,7 +486,9 @@ def measure_e2e(args, wl, prob, dev, stream, last, q_d, k_d, x_d):
         if a.dtype == np.uint16:
             return torch.from_numpy(a.view(np.int16)).view(torch.bfloat16).pin_memory()
         return torch.from_numpy(a).pin_memory()
-    qh, kh, xh = pin(wl.q), pin(wl.k), pin(wl.x)
+    qh, kh, xh = pin(wl.q if rows is None else rows[1]), pin(wl.k), pin(wl.x)
+    if rows is not None:
+        q_d = rows[2]
     nkeep = int(wl.cu_keep[-1])
     idx_h = torch.empty(nkeep, dtype=torch.int32).pin_memory()
     xs_h = torch.empty((nkeep, wl.feat_dim), dtype=xh.dtype).pin_memory()
@@ -454,7 +502,13 @@ def measure_e2e(args, wl, prob, dev, stream, last, q_d, k_d, x_d):
         q_d.copy_(qh, non_blocking=True)
         k_d.copy_(kh, non_blocking=True)
         x_d.copy_(xh, non_blocking=True)
-        if args.selector == "topk":
+        if rows is not None:
+            last.last_scores_rows(prob, rows[0], q_d, k_d, w_d, rows[3], stream)
+            if args.selector == "topk":
+                last.last_select_topk(prob, w_d, idx_d, ws, stream, x=x_d, x_out=xs_d)
+            else:
+                last.last_select(prob, w_d, x_d, idx_d, ws, stream, x_out=xs_d)
+        elif args.selector == "topk":
             last.last_scores(prob, q_d, k_d, w_d, ws, stream)
             last.last_select_topk(prob, w_d, idx_d, ws, stream, x=x_d, x_out=xs_d)
         else:

@@ -3,19 +3,22 @@
 //
 // Request b has M_b query rows at positions row_pos (after its visual span); row m
 // sees the keys 0 .. row_pos[m] (causal softmax, Eq. 6).  Scores are summed over
-// rows, layers and q-heads at the visual positions and normalised (Eq. 8).
+// rows, layers and q-heads at the visual positions and normalised (Eq. 8).  A
+// "column" is one (row, q-head of kv-head g) pair: G = Hq / Hkv columns per row.
 //
-// rows_logits_kernel: one CTA of 128 threads per (request, 128-key chunk, layer,
-//   kv-head g).  The chunk's keys of g (A, M = 128) and the request's query rows of
-//   the G q-heads of g (B, N = M_b * G padded to a multiple of 16) are staged in
-//   shared memory in the K-major 128-byte-swizzled layout; one thread issues
-//   tcgen05.mma (bf16, fp32 accumulator in TMEM) over D / 64 K blocks.  Thread t
-//   owns key t (TMEM lane t): per column (row, head) it masks keys past the row's
-//   position, and the CTA reduces the column's max and its sums of 2^(z - max) over
-//   all and over the visual keys (log2 domain), and writes the visual logits.
-// rows_tokens_kernel: one CTA per (request, 256 visual tokens): merges each
-//   (row, layer, head)'s chunk statistics in chunk order and sums the visual
-//   tokens' probabilities over them, divided by the total visual mass.
+// Four launches, all deterministic (fixed reduction orders, no float atomics):
+// rows_stats_kernel (request, 128-key chunk, layer, kv-head, 128-column tile):
+//   tcgen05.mma with the query columns as M and the chunk's keys as N (bf16, fp32
+//   accumulator in TMEM); thread t owns column t and takes, over its TMEM lane, the
+//   masked max of its logits (log2 domain) and the sums of 2^(z - max) over all and
+//   over the visual keys -- the chunk statistics of Eq. 6's softmax.
+// rows_merge_kernel (request): merges each column's chunk statistics in chunk
+//   order into (max, 1/Z) and the request's visual probability mass.
+// rows_probs_kernel (request, visual 128-key chunk, layer, kv-head): the same
+//   contraction with the keys as M; thread t owns key t and sums the probabilities
+//   2^(z - max) / Z over the columns (every column sees every visual key).
+// rows_final_kernel (request, 256 visual tokens): adds the (layer, kv-head)
+//   partial sums and divides by the visual mass (Eq. 7-8).
 #include "last_device.cuh"
 #include "last_internal.h"
 
@@ -29,242 +32,276 @@ namespace last {
 
 namespace {
 
-// Per-request metadata (int32 slots; the two 64-bit offsets take two slots each
-// and sit 8-byte aligned since a row is 12 slots).
+// Per-request metadata (int32 slots; the 64-bit statistics offset takes two slots
+// and sits 8-byte aligned since a row is 12 slots).
 enum RowsField : int {
   kRSeqStart = 0, kRSeqLen, kRVisStart, kRVisOff, kRNumVis, kRRowOff, kRNumRows,
-  kRNumChunks, kRStatBase = 8, kRZlogBase = 10, kRowsFields = 12
+  kRNumChunks, kRStatBase = 8, kRCoefBase = 10, kRowsFields = 12
 };
 
-constexpr int kRowsChunk = 128;     // keys per CTA (MMA M)
-constexpr int kRowsThreads = 128;
-constexpr int kRowsMaxN = 256;      // query rows x heads per kv-head (MMA N)
-constexpr int kRowsMaxRH = 6144;    // (row, layer, head) triples per request
+constexpr int kRowsChunk = 128;     // keys per CTA
+constexpr int kRowsThreads = 128;   // one thread per TMEM lane
+constexpr int kRowsMaxN = 256;      // columns (rows x G) per request
+constexpr int kRowsMaxRH = 6144;    // (row, layer, q-head) triples per request
 
 struct RowsArgs {
   const __nv_bfloat16 *q, *k;
   const int32_t *meta;
-  const int2 *items;
+  const int2 *items1, *items2;
   const int32_t *row_pos;
-  float4 *stats;
-  float *zlog;
+  float4 *stats;         // per column-layer-head triple x chunk: max, sum, visual sum
+  float2 *coef;          // per triple: max, 1 / Z
+  float *inv_total;      // per request: 1 / visual mass
+  float *partial;        // [L][Hkv][total_vis] probability sums
   float *w;
-  long long total_keys;
+  long long total_keys, total_vis;
   int L, Hq, Hkv, D, G, npad;
-  uint32_t tmem_cols;
+  uint32_t tmem_stats, tmem_probs;
   float qscale;          // softmax scale * log2(e)
   unsigned *err;
 };
 
+__device__ __forceinline__ long long stat_base(const int32_t *m) {
+  return *reinterpret_cast<const long long *>(m + kRStatBase);
+}
+
+// 16-byte chunk j of row `row` of a K-major operand with 128-byte rows and the
+// 128-byte swizzle; K blocks of `rows` rows each.
+__device__ __forceinline__ unsigned char *sw128_chunk(unsigned char *base, int rows, int row, int j) {
+  return base + (j >> 3) * (rows * 128) + row * 128 + (((j & 7) ^ (row & 7)) << 4);
+}
+
+// Keys c*128 .. c*128+127 of kv-head g (zero past P) into a 128-row operand.
+__device__ __forceinline__ void stage_keys(unsigned char *dst, const RowsArgs &a, int seq0, int P,
+                                           int c, int l, int g) {
+  const int t = threadIdx.x, p = c * kRowsChunk + t;
+  const __nv_bfloat16 *src = a.k + (((long long)l * a.total_keys + seq0 + p) * a.Hkv + g) * a.D;
+  for (int j = 0; j < a.D / 8; ++j)
+    *reinterpret_cast<U4 *>(sw128_chunk(dst, kRowsChunk, t, j)) =
+        p < P ? ldg(src + 8 * j) : U4{0, 0, 0, 0};
+}
+
+// Query columns n0 .. n0+rows-1 (row n / G, q-head g*G + n % G; zero past ncol).
+__device__ __forceinline__ void stage_queries(unsigned char *dst, const RowsArgs &a, int rows,
+                                              int n0, int ncol, int row0, int l, int g) {
+  for (int idx = threadIdx.x; idx < rows * (a.D / 8); idx += kRowsThreads) {
+    const int i = idx / (a.D / 8), j = idx - i * (a.D / 8), n = n0 + i;
+    U4 v = U4{0, 0, 0, 0};
+    if (n < ncol) {
+      const int r = n / a.G, gg = n - r * a.G;
+      v = ldg(a.q + (((long long)(row0 + r) * a.L + l) * a.Hq + g * a.G + gg) * a.D + 8 * j);
+    }
+    *reinterpret_cast<U4 *>(sw128_chunk(dst, rows, i, j)) = v;
+  }
+}
+
+// D[tmem] = A[128 x D] * B[n x D]^T over D / 64 K blocks, one thread; completion on bar.
+__device__ __forceinline__ void rows_mma(uint32_t tmem, unsigned char *A, unsigned char *B, int n,
+                                         int nkb, unsigned long long *bar) {
+  const uint32_t idesc = umma_idesc_bf16(kRowsChunk, n);
+  for (int kb = 0; kb < nkb; ++kb)
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+      umma_bf16(tmem, umma_desc_sw128(smem_addr(A + kb * (kRowsChunk * 128)) + k * 32),
+                umma_desc_sw128(smem_addr(B + kb * (n * 128)) + k * 32), idesc, (kb | k) != 0 ? 1u : 0u);
+  umma_commit(bar);
+}
+
 }  // namespace
 
 __global__ void __launch_bounds__(kRowsThreads)
-rows_logits_kernel(const RowsArgs a) {
+rows_stats_kernel(const RowsArgs a) {
+  const int2 item = a.items1[blockIdx.x];
+  const int b = item.x, c = item.y, l = blockIdx.y;
+  const int g = blockIdx.z % a.Hkv, mt = blockIdx.z / a.Hkv;
+  const int32_t *m = a.meta + b * kRowsFields;
+  const int ncol = m[kRNumRows] * a.G;
+  if (mt * kRowsThreads >= ncol) return;   // the whole CTA leaves before any allocation
   extern __shared__ __align__(16) unsigned char smem_raw[];
   unsigned char *smem = reinterpret_cast<unsigned char *>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   const int nkb = a.D / 64;
-  const int npad = a.npad;
-  unsigned char *sA = smem;                                   // nkb x [128 keys][128 B]
-  unsigned char *sB = smem + nkb * kRowsChunk * 128;          // nkb x [npad rows][128 B]
-  float *red = reinterpret_cast<float *>(sB + (size_t)nkb * npad * 128);   // [4][16] x 2
-  float *colv = red + 2 * 4 * 16;                              // [16] column max
-  unsigned long long *bar = reinterpret_cast<unsigned long long *>(colv + 16);
+  unsigned char *sQ = smem, *sK = smem + nkb * (kRowsChunk * 128);
+  unsigned long long *bar = reinterpret_cast<unsigned long long *>(sK + nkb * (kRowsChunk * 128));
   uint32_t *tslot = reinterpret_cast<uint32_t *>(bar + 1);
+  const int seq0 = m[kRSeqStart], P = m[kRSeqLen], v0 = m[kRVisStart], nvis = m[kRNumVis];
+  const int row0 = m[kRRowOff], nch = m[kRNumChunks];
+  const int t = threadIdx.x, warp = t >> 5;
 
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int2 item = a.items[blockIdx.x];
-  const int b = item.x, c = item.y, l = blockIdx.y, g = blockIdx.z;
-  const int32_t *m = a.meta + b * kRowsFields;
-  const int seq0 = m[kRSeqStart], P = m[kRSeqLen], v0 = m[kRVisStart];
-  const int nvis = m[kRNumVis], row0 = m[kRRowOff], nrows = m[kRNumRows];
-  const int nch = m[kRNumChunks];
-  const long long sbase = ((const long long *)(m + kRStatBase))[0];
-  const long long zbase = ((const long long *)(m + kRZlogBase))[0];
-  const int G = a.G, ncol = nrows * G;
-
-  if (tid == 0) {
+  if (t == 0) {
     mbar_init(bar, 1);
     fence_mbar_init();
   }
-  if (warp == 0) tmem_alloc(tslot, a.tmem_cols);
+  if (warp == 0) tmem_alloc(tslot, a.tmem_stats);
+  stage_queries(sQ, a, kRowsThreads, mt * kRowsThreads, ncol, row0, l, g);
+  stage_keys(sK, a, seq0, P, c, l, g);
+  fence_proxy_async_smem();
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tslot;
+  if (t == 0) rows_mma(tmem, sQ, sK, kRowsChunk, nkb, bar);
+  __syncwarp();
+  mbar_wait_bounded(bar, 0, a.err, kErrTimeout);
+  tc_fence_after();
 
-  // A: key t of the chunk, 16-byte chunk j -> K block j / 8, row t, swizzled column
-  {
-    const int p = c * kRowsChunk + tid;
-    const __nv_bfloat16 *src = a.k + (((long long)l * a.total_keys + seq0 + p) * a.Hkv + g) * a.D;
-    for (int j = 0; j < a.D / 8; ++j) {
-      const U4 v = p < P ? ldg(src + 8 * j) : U4{0, 0, 0, 0};
-      *reinterpret_cast<U4 *>(sA + (j >> 3) * (kRowsChunk * 128) + tid * 128 +
-                              (((j & 7) ^ (tid & 7)) << 4)) = v;
+  // column n: its row's position bounds the keys it sees
+  const int n = mt * kRowsThreads + t;
+  const bool col_ok = n < ncol;
+  const int r = col_ok ? n / a.G : 0;
+  const int pos = col_ok ? a.row_pos[row0 + r] : -1;
+  const uint32_t lane_addr = tmem + ((uint32_t)(32 * warp) << 16);
+  const int p0 = c * kRowsChunk;
+  float mx = -INFINITY;
+  for (int j0 = 0; j0 < kRowsChunk; j0 += 16) {
+    uint32_t raw[16];
+    tmem_ld16(lane_addr + (uint32_t)j0, raw);
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      const int p = p0 + j0 + j;
+      if (p < P && p <= pos) mx = fmaxf(mx, __uint_as_float(raw[j]) * a.qscale);
     }
   }
-  // B: column n = (row n / G, head g * G + n % G)
-  for (int idx = tid; idx < npad * (a.D / 8); idx += kRowsThreads) {
-    const int n = idx / (a.D / 8), j = idx - n * (a.D / 8);
-    U4 v = U4{0, 0, 0, 0};
-    if (n < ncol) {
-      const int r = n / G, gg = n - r * G;
-      v = ldg(a.q + (((long long)(row0 + r) * a.L + l) * a.Hq + g * G + gg) * a.D + 8 * j);
+  // (a column with no visible key in this chunk keeps max = -inf and adds nothing;
+  // the TMEM loads stay warp-uniform)
+  float sum = 0.f, vis = 0.f;
+  for (int j0 = 0; j0 < kRowsChunk; j0 += 16) {
+    uint32_t raw[16];
+    tmem_ld16(lane_addr + (uint32_t)j0, raw);
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      const int p = p0 + j0 + j;
+      if (p < P && p <= pos) {
+        const float e = exp2f(__uint_as_float(raw[j]) * a.qscale - mx);
+        sum += e;
+        if (p >= v0 && p < v0 + nvis) vis += e;
+      }
     }
-    *reinterpret_cast<U4 *>(sB + (j >> 3) * (npad * 128) + n * 128 + (((j & 7) ^ (n & 7)) << 4)) = v;
+  }
+  if (col_ok) {
+    const int h = g * a.G + (n - r * a.G);
+    const long long rh = ((long long)r * a.L + l) * a.Hq + h;
+    a.stats[stat_base(m) + rh * nch + c] = make_float4(mx, sum, vis, 0.f);
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) tmem_dealloc(tmem, a.tmem_stats);
+}
+
+__global__ void __launch_bounds__(1024)
+rows_merge_kernel(const RowsArgs a) {
+  __shared__ float red[32];
+  const int b = blockIdx.x;
+  const int32_t *m = a.meta + b * kRowsFields;
+  const int RH = m[kRNumRows] * a.L * a.Hq, nch = m[kRNumChunks], cb = m[kRCoefBase];
+  const float4 *stats = a.stats + stat_base(m);
+  float vis_mass = 0.f;
+  for (int rh = threadIdx.x; rh < RH; rh += blockDim.x) {
+    const float4 *st = stats + (long long)rh * nch;
+    float mx = -INFINITY;
+    for (int c = 0; c < nch; ++c) mx = fmaxf(mx, st[c].x);
+    float z = 0.f, vz = 0.f;
+    for (int c = 0; c < nch; ++c) {
+      const float4 v = st[c];
+      const float f = v.x == -INFINITY ? 0.f : exp2f(v.x - mx);   // chunks past the row
+      z += v.y * f;
+      vz += v.z * f;
+    }
+    a.coef[cb + rh] = make_float2(mx, 1.0f / z);
+    vis_mass += vz / z;
+  }
+  // fixed-tree block sum of the visual masses
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) vis_mass += __shfl_xor_sync(0xffffffffu, vis_mass, o);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = vis_mass;
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    float v = threadIdx.x < (int)(blockDim.x >> 5) ? red[threadIdx.x] : 0.f;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    if (threadIdx.x == 0) a.inv_total[b] = 1.0f / v;
+  }
+}
+
+__global__ void __launch_bounds__(kRowsThreads)
+rows_probs_kernel(const RowsArgs a) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  unsigned char *smem = reinterpret_cast<unsigned char *>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  const int nkb = a.D / 64, npad = a.npad;
+  unsigned char *sK = smem, *sQ = smem + nkb * (kRowsChunk * 128);
+  float2 *cf = reinterpret_cast<float2 *>(sQ + nkb * (npad * 128));
+  unsigned long long *bar = reinterpret_cast<unsigned long long *>(cf + kRowsMaxN);
+  uint32_t *tslot = reinterpret_cast<uint32_t *>(bar + 1);
+  const int2 item = a.items2[blockIdx.x];
+  const int b = item.x, c = item.y, l = blockIdx.y, g = blockIdx.z;
+  const int32_t *m = a.meta + b * kRowsFields;
+  const int seq0 = m[kRSeqStart], P = m[kRSeqLen], v0 = m[kRVisStart], nvis = m[kRNumVis];
+  const int voff = m[kRVisOff], row0 = m[kRRowOff], ncol = m[kRNumRows] * a.G;
+  const int cb = m[kRCoefBase];
+  const int t = threadIdx.x, warp = t >> 5;
+
+  if (t == 0) {
+    mbar_init(bar, 1);
+    fence_mbar_init();
+  }
+  if (warp == 0) tmem_alloc(tslot, a.tmem_probs);
+  stage_keys(sK, a, seq0, P, c, l, g);
+  stage_queries(sQ, a, npad, 0, ncol, row0, l, g);
+  for (int n = t; n < ncol; n += kRowsThreads) {
+    const int r = n / a.G, h = g * a.G + (n - r * a.G);
+    cf[n] = a.coef[cb + ((long long)r * a.L + l) * a.Hq + h];
   }
   fence_proxy_async_smem();
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tslot;
-
-  if (tid == 0) {
-    const uint32_t idesc = umma_idesc_bf16(kRowsChunk, npad);
-    for (int kb = 0; kb < nkb; ++kb)
-#pragma unroll
-      for (int k = 0; k < 4; ++k)
-        umma_bf16(tmem, umma_desc_sw128(smem_addr(sA + kb * (kRowsChunk * 128)) + k * 32),
-                  umma_desc_sw128(smem_addr(sB + kb * (npad * 128)) + k * 32), idesc,
-                  (kb | k) != 0 ? 1u : 0u);
-    umma_commit(bar);
-  }
+  if (t == 0) rows_mma(tmem, sK, sQ, npad, nkb, bar);
   __syncwarp();
   mbar_wait_bounded(bar, 0, a.err, kErrTimeout);
   tc_fence_after();
 
-  const int p = c * kRowsChunk + tid;                  // this thread's key
-  const bool key_ok = p < P;
-  const bool vis = p >= v0 && p < v0 + nvis;
+  const int p = c * kRowsChunk + t;
+  float s0 = 0.f, s1 = 0.f;
   for (int n0 = 0; n0 < ncol; n0 += 16) {
     uint32_t raw[16];
     tmem_ld16(tmem + ((uint32_t)(32 * warp) << 16) + (uint32_t)n0, raw);
-    float z[16];
-    bool use[16];
 #pragma unroll
-    for (int j = 0; j < 16; ++j) {
-      const int n = n0 + j;
-      const int pos = n < ncol ? a.row_pos[row0 + n / G] : -1;
-      use[j] = key_ok && n < ncol && p <= pos;
-      z[j] = use[j] ? __uint_as_float(raw[j]) * a.qscale : -INFINITY;
+    for (int j = 0; j < 16; j += 2) {
+      if (n0 + j < ncol)
+        s0 += exp2f(__uint_as_float(raw[j]) * a.qscale - cf[n0 + j].x) * cf[n0 + j].y;
+      if (n0 + j + 1 < ncol)
+        s1 += exp2f(__uint_as_float(raw[j + 1]) * a.qscale - cf[n0 + j + 1].x) * cf[n0 + j + 1].y;
     }
-    // column max over the 128 keys
-#pragma unroll
-    for (int j = 0; j < 16; ++j) {
-      float v = z[j];
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
-      if (lane == 0) red[warp * 16 + j] = v;
-    }
-    __syncthreads();
-    if (tid < 16)
-      colv[tid] = fmaxf(fmaxf(red[tid], red[16 + tid]), fmaxf(red[32 + tid], red[48 + tid]));
-    __syncthreads();
-    // sums of 2^(z - max) over all keys and over the visual keys
-#pragma unroll
-    for (int j = 0; j < 16; ++j) {
-      float e = use[j] ? exp2f(z[j] - colv[j]) : 0.f;
-      float ev = vis ? e : 0.f;
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) {
-        e += __shfl_xor_sync(0xffffffffu, e, o);
-        ev += __shfl_xor_sync(0xffffffffu, ev, o);
-      }
-      if (lane == 0) {
-        red[warp * 16 + j] = e;
-        red[64 + warp * 16 + j] = ev;
-      }
-    }
-    __syncthreads();
-    if (tid < 16 && n0 + tid < ncol) {
-      const int n = n0 + tid, r = n / G, h = g * G + (n - r * G);
-      const float s = (red[tid] + red[16 + tid]) + (red[32 + tid] + red[48 + tid]);
-      const float sv = (red[64 + tid] + red[80 + tid]) + (red[96 + tid] + red[112 + tid]);
-      const long long rh = ((long long)r * a.L + l) * a.Hq + h;
-      a.stats[sbase + rh * nch + c] = make_float4(colv[tid], s, sv, 0.f);
-    }
-    // visual logits
-    if (vis && key_ok) {
-#pragma unroll
-      for (int j = 0; j < 16; ++j) {
-        const int n = n0 + j;
-        if (n < ncol) {
-          const int r = n / G, h = g * G + (n - r * G);
-          const long long rh = ((long long)r * a.L + l) * a.Hq + h;
-          a.zlog[zbase + rh * nvis + (p - v0)] = z[j];
-        }
-      }
-    }
-    __syncthreads();   // red / colv are reused by the next column group
   }
+  // every column's row sits after the visual span, so each visual key is unmasked
+  if (p >= v0 && p < v0 + nvis && p < P)
+    a.partial[((long long)l * a.Hkv + g) * a.total_vis + voff + (p - v0)] = s0 + s1;
   tc_fence_before();
   __syncthreads();
-  if (warp == 0) tmem_dealloc(tmem, a.tmem_cols);
+  if (warp == 0) tmem_dealloc(tmem, a.tmem_probs);
 }
 
 __global__ void __launch_bounds__(kScoreThreads)
-rows_tokens_kernel(const RowsArgs a) {
-  extern __shared__ float coef[];     // [RH] max, [RH] 1/Z, [RH] V/Z
-  __shared__ float inv_total_s;
-  const int b = blockIdx.y, tile = blockIdx.x;
+rows_final_kernel(const RowsArgs a) {
+  const int b = blockIdx.y;
   const int32_t *m = a.meta + b * kRowsFields;
-  const int nvis = m[kRNumVis], voff = m[kRVisOff], nrows = m[kRNumRows], nch = m[kRNumChunks];
-  if (tile * kTokenTile >= nvis) return;
-  const long long sbase = ((const long long *)(m + kRStatBase))[0];
-  const long long zbase = ((const long long *)(m + kRZlogBase))[0];
-  const int RH = nrows * a.L * a.Hq;
-  float *cmax = coef, *cinv = coef + RH, *cvis = coef + 2 * RH;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  for (int rh = warp; rh < RH; rh += kScoreThreads / 32) {
-    const float4 *st = a.stats + sbase + (long long)rh * nch;
-    float mx = -INFINITY;
-    for (int cc = lane; cc < nch; cc += 32) mx = fmaxf(mx, st[cc].x);
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-    float z = 0.f, vz = 0.f;
-    for (int cc = lane; cc < nch; cc += 32) {
-      const float4 v = st[cc];
-      const float f = v.x == -INFINITY ? 0.f : exp2f(v.x - mx);   // chunks past the row
-      z += v.y * f;
-      vz += v.z * f;
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      z += __shfl_xor_sync(0xffffffffu, z, o);
-      vz += __shfl_xor_sync(0xffffffffu, vz, o);
-    }
-    if (lane == 0) {
-      cmax[rh] = mx;
-      cinv[rh] = 1.0f / z;
-      cvis[rh] = vz / z;
-    }
-  }
-  __syncthreads();
-  if (warp == 0) {
-    float t = 0.f;
-    for (int rh = lane; rh < RH; rh += 32) t += cvis[rh];
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
-    if (lane == 0) inv_total_s = 1.0f / t;
-  }
-  __syncthreads();
-  const int i = tile * kTokenTile + threadIdx.x;
-  if (i < nvis) {
-    const float *zl = a.zlog + zbase + i;
-    float s0 = 0.f, s1 = 0.f;
-    int rh = 0;
-    for (; rh + 2 <= RH; rh += 2) {
-      s0 += exp2f(zl[(long long)rh * nvis] - cmax[rh]) * cinv[rh];
-      s1 += exp2f(zl[(long long)(rh + 1) * nvis] - cmax[rh + 1]) * cinv[rh + 1];
-    }
-    if (rh < RH) s0 += exp2f(zl[(long long)rh * nvis] - cmax[rh]) * cinv[rh];
-    a.w[voff + i] = (s0 + s1) * inv_total_s;
-  }
+  const int i = blockIdx.x * kScoreThreads + threadIdx.x;
+  if (i >= m[kRNumVis]) return;
+  const long long tok = m[kRVisOff] + i;
+  float s = 0.f;
+  for (int lg = 0; lg < a.L * a.Hkv; ++lg) s += a.partial[(long long)lg * a.total_vis + tok];
+  a.w[tok] = s * a.inv_total[b];
 }
 
 namespace {
 
 struct RowsPlan {
-  int B = 0, L = 0, Hq = 0, Hkv = 0, D = 0, G = 0, npad = 0, max_vis = 0, max_rh = 0;
-  long long total_keys = 0, total_vis = 0, total_rows = 0, total_items = 0;
-  size_t off_meta = 0, off_items = 0, off_pos = 0, off_stats = 0, off_zlog = 0, total_bytes = 0;
-  size_t blob_bytes = 0;
+  int B = 0, L = 0, Hq = 0, Hkv = 0, D = 0, G = 0, npad = 0, mtiles = 0, max_vis = 0;
+  long long total_keys = 0, total_vis = 0, total_rows = 0, n_items1 = 0, n_items2 = 0;
+  size_t off_meta = 0, off_items1 = 0, off_items2 = 0, off_pos = 0, blob_bytes = 0;
+  size_t off_stats = 0, off_coef = 0, off_inv = 0, off_partial = 0, total_bytes = 0;
   std::vector<int32_t> blob;
   float scale = 0.f;
 };
@@ -300,7 +337,7 @@ last_status make_rows_plan(const last_problem *p, const int32_t *cu_rows, const 
   pl->D = p->head_dim; pl->G = pl->Hq / pl->Hkv;
   pl->scale = p->softmax_scale > 0.f ? p->softmax_scale : (float)(1.0 / std::sqrt((double)p->head_dim));
   int max_cols = 0;
-  long long stats = 0, zlog = 0;
+  long long stats = 0, rh_total = 0;
   for (int b = 0; b < B; ++b) {
     const int P = p->cu_seqlens[b + 1] - p->cu_seqlens[b];
     const int N = p->cu_vis[b + 1] - p->cu_vis[b];
@@ -318,39 +355,49 @@ last_status make_rows_plan(const last_problem *p, const int32_t *cu_rows, const 
     const long long rh = (long long)M * pl->L * pl->Hq;
     if (rh > kRowsMaxRH)
       return rows_fail(LAST_ERR_UNSUPPORTED, "rows x layers x q-heads must be <= 6144 per request");
-    pl->max_rh = std::max<int>(pl->max_rh, (int)rh);
     const int nch = (P + kRowsChunk - 1) / kRowsChunk;
     stats += rh * nch;
-    zlog += rh * N;
-    pl->total_items += nch;
+    rh_total += rh;
+    pl->n_items1 += nch;
+    if (N > 0)
+      pl->n_items2 += (p->vis_start[b] + N - 1) / kRowsChunk - p->vis_start[b] / kRowsChunk + 1;
     pl->max_vis = std::max(pl->max_vis, N);
   }
   if (max_cols > kRowsMaxN)
     return rows_fail(LAST_ERR_UNSUPPORTED, "query rows x (num_q_heads / num_kv_heads) must be <= 256");
+  if (rh_total > 0x7fffffffLL) return rows_fail(LAST_ERR_UNSUPPORTED, "too many query rows in all");
   pl->npad = std::max(16, (max_cols + 15) / 16 * 16);
+  pl->mtiles = (max_cols + kRowsThreads - 1) / kRowsThreads;
   pl->total_keys = p->cu_seqlens[B];
   pl->total_vis = p->cu_vis[B];
   pl->total_rows = cu_rows[B];
-  size_t o = 0;
-  o = alignr(o + 64);                       // error word
+  size_t o = alignr(64);                     // error word first
   pl->off_meta = o;
   o = alignr(o + sizeof(int32_t) * kRowsFields * std::max(B, 1));
-  pl->off_items = o;
-  o = alignr(o + sizeof(int32_t) * 2 * std::max<long long>(pl->total_items, 1));
+  pl->off_items1 = o;
+  o = alignr(o + sizeof(int32_t) * 2 * std::max<long long>(pl->n_items1, 1));
+  pl->off_items2 = o;
+  o = alignr(o + sizeof(int32_t) * 2 * std::max<long long>(pl->n_items2, 1));
   pl->off_pos = o;
   o = alignr(o + sizeof(int32_t) * std::max<long long>(pl->total_rows, 1));
   pl->blob_bytes = o;
   pl->off_stats = o;
   o = alignr(o + sizeof(float) * 4 * (size_t)std::max<long long>(stats, 1));
-  pl->off_zlog = o;
-  o = alignr(o + sizeof(float) * (size_t)std::max<long long>(zlog, 1));
+  pl->off_coef = o;
+  o = alignr(o + sizeof(float) * 2 * (size_t)std::max<long long>(rh_total, 1));
+  pl->off_inv = o;
+  o = alignr(o + sizeof(float) * std::max(B, 1));
+  pl->off_partial = o;
+  o = alignr(o + sizeof(float) * (size_t)pl->L * pl->Hkv * (size_t)std::max<long long>(pl->total_vis, 1));
   pl->total_bytes = o;
-  // staging blob: [error word][meta][items][row positions]
+  // staging blob: [error word][meta][items of every chunk][items of visual chunks][positions]
   pl->blob.assign(pl->blob_bytes / sizeof(int32_t), 0);
   int32_t *meta = pl->blob.data() + pl->off_meta / 4;
-  int32_t *items = pl->blob.data() + pl->off_items / 4;
+  int32_t *it1 = pl->blob.data() + pl->off_items1 / 4;
+  int32_t *it2 = pl->blob.data() + pl->off_items2 / 4;
   int32_t *pos = pl->blob.data() + pl->off_pos / 4;
-  long long sb = 0, zb = 0, it = 0;
+  long long sb = 0, i1 = 0, i2 = 0;
+  int cb = 0;
   for (int b = 0; b < B; ++b) {
     int32_t *mm = meta + b * kRowsFields;
     const int P = p->cu_seqlens[b + 1] - p->cu_seqlens[b];
@@ -365,18 +412,31 @@ last_status make_rows_plan(const last_problem *p, const int32_t *cu_rows, const 
     mm[kRRowOff] = cu_rows[b];
     mm[kRNumRows] = M;
     mm[kRNumChunks] = nch;
-    std::memcpy(mm + kRStatBase, &sb, sizeof sb);   // 64-bit offsets in two int32 slots
-    std::memcpy(mm + kRZlogBase, &zb, sizeof zb);
-    const long long rh = (long long)M * pl->L * pl->Hq;
-    sb += rh * nch;
-    zb += rh * N;
-    for (int c = 0; c < nch; ++c, ++it) {
-      items[2 * it] = b;
-      items[2 * it + 1] = c;
+    std::memcpy(mm + kRStatBase, &sb, sizeof sb);   // 64-bit offset in two int32 slots
+    mm[kRCoefBase] = cb;
+    const int rh = M * pl->L * pl->Hq;
+    sb += (long long)rh * nch;
+    cb += rh;
+    for (int c = 0; c < nch; ++c, ++i1) {
+      it1[2 * i1] = b;
+      it1[2 * i1 + 1] = c;
     }
+    if (N > 0)
+      for (int c = p->vis_start[b] / kRowsChunk; c <= (p->vis_start[b] + N - 1) / kRowsChunk; ++c, ++i2) {
+        it2[2 * i2] = b;
+        it2[2 * i2 + 1] = c;
+      }
   }
   for (long long r = 0; r < pl->total_rows; ++r) pos[r] = row_pos[r];
   return LAST_OK;
+}
+
+// Dynamic shared memory of a 128-thread kernel holding `cols` TMEM columns: the
+// operands, and at least enough that at most 512 / cols CTAs share an SM, so every
+// CTA's TMEM allocation is granted at once.
+size_t tmem_safe_smem(size_t operands, uint32_t cols) {
+  const size_t per_sm = 228 * 1024;
+  return std::max(operands, per_sm / (512 / cols + 1) + 1);
 }
 
 }  // namespace
@@ -420,39 +480,49 @@ extern "C" last_status last_scores_rows(const last_problem *p, const int32_t *cu
   a.q = static_cast<const __nv_bfloat16 *>(q_rows);
   a.k = static_cast<const __nv_bfloat16 *>(k);
   a.meta = reinterpret_cast<const int32_t *>(wsc + pl.off_meta);
-  a.items = reinterpret_cast<const int2 *>(wsc + pl.off_items);
+  a.items1 = reinterpret_cast<const int2 *>(wsc + pl.off_items1);
+  a.items2 = reinterpret_cast<const int2 *>(wsc + pl.off_items2);
   a.row_pos = reinterpret_cast<const int32_t *>(wsc + pl.off_pos);
   a.stats = reinterpret_cast<float4 *>(wsc + pl.off_stats);
-  a.zlog = reinterpret_cast<float *>(wsc + pl.off_zlog);
+  a.coef = reinterpret_cast<float2 *>(wsc + pl.off_coef);
+  a.inv_total = reinterpret_cast<float *>(wsc + pl.off_inv);
+  a.partial = reinterpret_cast<float *>(wsc + pl.off_partial);
   a.w = w_out;
   a.total_keys = pl.total_keys;
+  a.total_vis = pl.total_vis;
   a.L = pl.L; a.Hq = pl.Hq; a.Hkv = pl.Hkv; a.D = pl.D; a.G = pl.G; a.npad = pl.npad;
-  uint32_t tcols = 32;
-  while ((int)tcols < pl.npad) tcols *= 2;
-  a.tmem_cols = tcols;
+  a.tmem_stats = 128;
+  uint32_t tp = 32;
+  while ((int)tp < pl.npad) tp *= 2;
+  a.tmem_probs = tp;
   a.qscale = pl.scale * 1.4426950408889634f;
   a.err = reinterpret_cast<unsigned *>(wsc);
+  auto fail_launch = [](cudaError_t err, const char *what) {
+    return rows_fail(LAST_ERR_CUDA, std::string(what) + ": " + cudaGetErrorString(err));
+  };
 
-  // Shared memory: the operands, plus enough that at most 512 / tmem_cols CTAs share
-  // an SM, so every CTA's TMEM allocation is granted at once.
   const int nkb = pl.D / 64;
-  size_t smem = 1024 + (size_t)nkb * kRowsChunk * 128 + (size_t)nkb * pl.npad * 128 + 1024;
-  const size_t per_sm = 228 * 1024;
-  const size_t floor_smem = per_sm / (512 / tcols + 1) + 1;
-  smem = std::max(smem, floor_smem);
-  e = cudaFuncSetAttribute(rows_logits_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  if (e != cudaSuccess) return rows_fail(LAST_ERR_CUDA, std::string("rows logits: ") + cudaGetErrorString(e));
-  rows_logits_kernel<<<dim3((unsigned)pl.total_items, pl.L, pl.Hkv), kRowsThreads, smem, s>>>(a);
-  if ((e = cudaGetLastError()) != cudaSuccess)
-    return rows_fail(LAST_ERR_CUDA, std::string("rows logits launch: ") + cudaGetErrorString(e));
-  const size_t tsmem = sizeof(float) * 3 * pl.max_rh;
-  if (tsmem > 48 * 1024) {
-    e = cudaFuncSetAttribute(rows_tokens_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)tsmem);
-    if (e != cudaSuccess) return rows_fail(LAST_ERR_CUDA, std::string("rows tokens: ") + cudaGetErrorString(e));
+  const size_t op = 1024 + (size_t)2 * nkb * kRowsChunk * 128 + 64;
+  const size_t smem1 = tmem_safe_smem(op, a.tmem_stats);
+  if ((e = cudaFuncSetAttribute(rows_stats_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)smem1)) != cudaSuccess)
+    return fail_launch(e, "rows stats");
+  rows_stats_kernel<<<dim3((unsigned)pl.n_items1, pl.L, pl.Hkv * pl.mtiles), kRowsThreads, smem1, s>>>(a);
+  if ((e = cudaGetLastError()) != cudaSuccess) return fail_launch(e, "rows stats launch");
+  rows_merge_kernel<<<pl.B, 1024, 0, s>>>(a);
+  if ((e = cudaGetLastError()) != cudaSuccess) return fail_launch(e, "rows merge launch");
+  if (pl.n_items2 > 0) {
+    const size_t op2 = 1024 + (size_t)nkb * kRowsChunk * 128 + (size_t)nkb * pl.npad * 128 +
+                       sizeof(float2) * kRowsMaxN + 64;
+    const size_t smem2 = tmem_safe_smem(op2, a.tmem_probs);
+    if ((e = cudaFuncSetAttribute(rows_probs_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  (int)smem2)) != cudaSuccess)
+      return fail_launch(e, "rows probs");
+    rows_probs_kernel<<<dim3((unsigned)pl.n_items2, pl.L, pl.Hkv), kRowsThreads, smem2, s>>>(a);
+    if ((e = cudaGetLastError()) != cudaSuccess) return fail_launch(e, "rows probs launch");
   }
-  const int tiles = (pl.max_vis + kTokenTile - 1) / kTokenTile;
-  rows_tokens_kernel<<<dim3(tiles, pl.B), kScoreThreads, tsmem, s>>>(a);
-  if ((e = cudaGetLastError()) != cudaSuccess)
-    return rows_fail(LAST_ERR_CUDA, std::string("rows tokens launch: ") + cudaGetErrorString(e));
+  const int tiles = (pl.max_vis + kScoreThreads - 1) / kScoreThreads;
+  rows_final_kernel<<<dim3(tiles, pl.B), kScoreThreads, 0, s>>>(a);
+  if ((e = cudaGetLastError()) != cudaSuccess) return fail_launch(e, "rows final launch");
   return LAST_OK;
 }

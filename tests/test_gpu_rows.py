@@ -4,7 +4,7 @@ import numpy as np
 import pytest
 
 import oracle
-from workloads import config, custom, f32_to_bf16_bits
+from workloads import config, custom, query_rows
 
 from gpu_util import SCORE_ATOL, SCORE_RTOL, problem_of, to_dev
 
@@ -24,33 +24,9 @@ def _built():
 
 
 def make_rows(wl, source, rng, m_rows=8):
-    """Query positions after each request's visual span: First, Middle and Last of
-    the text rows, or up to m_rows of them (All Mean); one random bf16 query vector
-    per row, layer and q-head (the last row takes the workload's own p* query)."""
-    cu, pos = [0], []
-    for b in range(wl.batch):
-        P = int(wl.cu_seqlens[b + 1] - wl.cu_seqlens[b])
-        first = int(wl.vis_start[b] + (wl.cu_vis[b + 1] - wl.cu_vis[b]))
-        text = np.arange(first, P)
-        if source == "first":
-            sel = text[:1]
-        elif source == "middle":
-            sel = text[(len(text) - 1) // 2:][:1]
-        elif source == "last":
-            sel = text[-1:]
-        else:
-            sel = text[np.linspace(0, len(text) - 1, min(m_rows, len(text))).round().astype(int)]
-            sel = np.unique(sel)
-        pos += sel.tolist()
-        cu.append(len(pos))
-    R = len(pos)
-    q = rng.standard_normal((R, wl.num_layers, wl.num_q_heads, wl.head_dim)).astype(np.float32)
-    q = f32_to_bf16_bits(q)
-    for b in range(wl.batch):                  # a row at p* uses the request's own query
-        for r in range(cu[b], cu[b + 1]):
-            if pos[r] == int(wl.cu_seqlens[b + 1] - wl.cu_seqlens[b]) - 1:
-                q[r] = wl.q[b]
-    return np.array(cu, np.int32), np.array(pos, np.int32), q
+    """Query rows of the given source (First, Middle, Last or All Mean over up to
+    m_rows text rows), seeded from rng."""
+    return query_rows(wl, source, m_rows=m_rows, seed=int(rng.integers(1 << 30)))
 
 
 def run_rows(wl, cu, pos, q):

@@ -6,7 +6,7 @@ aggregation, no selection), and both the oracle-side tests and the CUDA-side
 tests/benchmark draw their inputs from it.
 """
 from .synth import (Workload, bf16_bits_to_f32, config, custom, f32_to_bf16_bits,
-                    CONFIG_NAMES)
+                    query_rows, CONFIG_NAMES)
 
 __all__ = ["Workload", "bf16_bits_to_f32", "config", "custom", "f32_to_bf16_bits",
-           "CONFIG_NAMES"]
+           "query_rows", "CONFIG_NAMES"]

@@ -269,3 +269,38 @@ def config(name: str, *, budget=None, batch=None, n_vis=None, seed=None) -> Work
                       dtype="bf16", keep_frac=pct, n_planted=10, video_frame=512,
                       video_sigma=0.05, note="32 frames x 512, random-walk frames")
     raise ValueError(f"unknown workload {name!r}")
+
+
+def query_rows(wl: Workload, source: str, m_rows: int = 32, seed: int = 7):
+    """Query rows for Table 4's attention sources: positions after each request's
+    visual span (its text rows) -- the first ("first"), the middle ("middle"), the
+    last ("last", p* = P_b - 1) or up to m_rows spread evenly over them ("all") --
+    and one query vector per row, layer and q-head drawn like the workload's q (a
+    row at p* takes the request's own p* query).  Returns (cu_rows, row_pos, q_rows)
+    with q_rows [sum M][L][Hq][D] in the workload's dtype."""
+    cu, pos = [0], []
+    for b in range(wl.batch):
+        P = int(wl.cu_seqlens[b + 1] - wl.cu_seqlens[b])
+        first = int(wl.vis_start[b] + (wl.cu_vis[b + 1] - wl.cu_vis[b]))
+        text = np.arange(first, P)
+        if source == "first":
+            sel = text[:1]
+        elif source == "middle":
+            sel = text[(len(text) - 1) // 2:][:1]
+        elif source == "last":
+            sel = text[-1:]
+        elif source == "all":
+            sel = np.unique(text[np.linspace(0, len(text) - 1, min(m_rows, len(text)))
+                                 .round().astype(int)])
+        else:
+            raise ValueError(f"unknown attention source {source!r}")
+        pos += sel.tolist()
+        cu.append(len(pos))
+    rng = _rng(seed, 99)
+    q = rng.standard_normal((len(pos), wl.num_layers, wl.num_q_heads, wl.head_dim)).astype(np.float32)
+    q = _cast(q * np.float32(1.0 / math.sqrt(wl.head_dim)), wl.dtype)   # q ~ N(0, 1)/sqrt(D)
+    for b in range(wl.batch):
+        for r in range(cu[b], cu[b + 1]):
+            if pos[r] == int(wl.cu_seqlens[b + 1] - wl.cu_seqlens[b]) - 1:
+                q[r] = wl.q[b]
+    return np.array(cu, np.int32), np.array(pos, np.int32), np.ascontiguousarray(q)
