@@ -85,7 +85,8 @@ struct SelectArgs {
 // Shared-memory carve-up, identical on host (sizing) and device.
 struct SelectSmem {
   size_t aring, xcache, cbuf, ring, blk, w, r, dl, list, sel, wtop, pub_key, pub_f, lp_key,
-      lp_f, lp_idx, lp_row, pair, acc, misc, bar, cnt, tbar, tslot, fidx, fmask, fcnt, total;
+      lp_f, lp_idx, lp_row, pair, acc, misc, bar, cnt, tbar, tslot, fidx, fmask, fcnt, gram, plist,
+      total;
 };
 // K blocks of kTcBK elements covering a feature row.
 __host__ __device__ inline int tc_kblocks(int dv) { return (dv + kTcBK - 1) / kTcBK; }
@@ -137,11 +138,13 @@ __host__ __device__ inline SelectSmem select_smem(int cache_rows, int row_bytes,
   s.bar = o; o += sizeof(unsigned long long);
   s.cnt = o; o += sizeof(int) * kMaxCluster;
   o = align16(o);
-  s.tbar = o; o += tc ? sizeof(unsigned long long) * (2 * kTcMaxStages + 1) : 0;
+  s.tbar = o; o += tc ? sizeof(unsigned long long) * (2 * kTcMaxStages + 2) : 0;
   s.tslot = o; o += tc ? 16 : 0;
   s.fidx = o; o += tc ? align16(sizeof(int) * tpc_max) : 0;
   s.fmask = o; o += tc ? align16(sizeof(uint32_t) * tpc_max) : 0;
   s.fcnt = o; o += tc ? 16 : 0;
+  s.gram = o; o += tc ? sizeof(float) * kLcap * kLcap : 0;       // list Gram (tensor cores)
+  s.plist = o; o += tc ? align16(sizeof(int) * (kMaxPairs + 1)) : 0;   // pairs to evaluate
   s.total = align16(o) + 1024;   // slack for aligning the base to 1024 bytes
   return s;
 }
@@ -287,6 +290,7 @@ select_kernel(const __grid_constant__ SelectArgs a) {
   const int nstage = TC ? a.tc_stages : 1;
   unsigned long long *tempty = tfull + kTcMaxStages;
   unsigned long long *tdone = tempty + kTcMaxStages;
+  unsigned long long *tpair = tdone + 1;
   if (threadIdx.x == 0) {
     mbar_init(bar, 1);
     if constexpr (TC) {
@@ -295,6 +299,7 @@ select_kernel(const __grid_constant__ SelectArgs a) {
         mbar_init(&tempty[i], 1);
       }
       mbar_init(tdone, 1);
+      mbar_init(tpair, 1);
     }
     fence_mbar_init();
   }
@@ -614,6 +619,7 @@ select_kernel(const __grid_constant__ SelectArgs a) {
     // pair is recomputed in the canonical order.  delta thus stays bit-identical
     // to the CUDA-core update.
     uint32_t tc_pit = 0, tc_mit = 0, tc_dph = 0;   // producer / MMA / done phase counters
+    uint32_t tc_pph = 0;                            // list-Gram phase
     // After one expired wait every later tensor-core wait returns at once, so a
     // broken call ends quickly (reporting LAST_ERR_TIMEOUT) instead of waiting out
     // each limit in turn.
@@ -912,14 +918,87 @@ select_kernel(const __grid_constant__ SelectArgs a) {
       wait_rows();
       __syncthreads();
       // pairwise dots of L, split over the cluster (4 interleaved pairs per warp),
-      // broadcast to every CTA
+      // broadcast to every CTA.  With the tensor-core update the list's Gram is first
+      // taken on the tensor cores: a pair whose tensor-core distance is at least
+      // tc_eps above both members' delta can lower neither member's delta during the
+      // replay (delta only shrinks), so its dot is stored as -inf (distance +inf) and
+      // only the other pairs are evaluated in the canonical order.
       {
         const int npairs = nL * (nL - 1) / 2;
-        for (int p0 = ((int)rank + C * warp) * 4; p0 < npairs; p0 += C * kSelectWarps * 4) {
+        int nwork = npairs;              // pairs evaluated exactly
+        int *plist = reinterpret_cast<int *>(smem + S.plist);
+        if constexpr (TC) {
+          float *gram = reinterpret_cast<float *>(smem + S.gram);
+          fence_proxy_async_smem();
+          tc_fence_before();
+          __syncthreads();
+          tc_fence_after();
+          const uint32_t gcol = (uint32_t)(((a.tpc_max + kTcBM - 1) / kTcBM) * lcap);
+          if (threadIdx.x == 32) {
+            const uint32_t idesc = umma_idesc_bf16(kTcBM, lcap);
+            const int nkb = tc_kblocks(dv);
+            for (int kb = 0; kb < nkb; ++kb)
+#pragma unroll
+              for (int k = 0; k < kTcBK / 16; ++k)
+                umma_bf16(tmem + gcol, umma_desc_sw128(cbuf_sa + kb * lcap * 128 + k * 32),
+                          umma_desc_sw128(cbuf_sa + kb * lcap * 128 + k * 32), idesc,
+                          (kb | k) != 0 ? 1u : 0u);
+            umma_commit(tpair);
+          }
+          __syncwarp();
+          twait(tpair, tc_pph);
+          tc_pph ^= 1u;
+          tc_fence_after();
+          if (warp == 0) {   // TMEM lanes 0..31 and the columns: cbuf rows
+            for (int v0 = 0; v0 < lcap; v0 += 16) {
+              uint32_t raw[16];
+              tmem_ld16(tmem + gcol + (uint32_t)v0, raw);
+#pragma unroll
+              for (int j = 0; j < 16; ++j)
+                if (lane < lcap) gram[lane * kLcap + v0 + j] = __uint_as_float(raw[j]);
+            }
+          }
+          tc_fence_before();
+          __syncthreads();
+          // pairs that still need the canonical dot, compacted in pair order
+          int base = 0;
+          for (int q0 = 0; q0 < npairs; q0 += kSelThreads) {
+            const int p = q0 + (int)threadIdx.x;
+            bool need = false;
+            if (p < npairs) {
+              int u = 0, rem = p;
+              while (rem >= nL - 1 - u) { rem -= nL - 1 - u; ++u; }
+              const int v = u + 1 + rem;
+              const float ru = lp_f[u * 3 + 2], rv = lp_f[v * 3 + 2];
+              const float du = lp_f[u * 3 + 0], dv_ = lp_f[v * 3 + 0];
+              const float g = gram[lp_row[u] * kLcap + lp_row[v]];
+              const float d = __fsub_rn(1.0f, __fmul_rn(__fmul_rn(g, ru), rv));
+              need = ru == 0.f || rv == 0.f || !(__fsub_rn(d, a.tc_eps) >= fmaxf(du, dv_));
+              if (!need) pairbuf[par * kMaxPairs + p] = -INFINITY;
+            }
+            const unsigned bal = __ballot_sync(0xffffffffu, need);
+            if (lane == 0) cnt_s[warp] = __popc(bal);   // scratch: cnt_s is idle until the epilogue
+            __syncthreads();
+            int off = base, tot = 0;
+#pragma unroll
+            for (int w8 = 0; w8 < kSelectWarps; ++w8) {
+              off += w8 < warp ? cnt_s[w8] : 0;
+              tot += cnt_s[w8];
+            }
+            if (need) plist[off + __popc(bal & ((1u << lane) - 1u))] = p;
+            base += tot;
+            __syncthreads();
+          }
+          nwork = base;
+        }
+        for (int p0 = ((int)rank + C * warp) * 4; p0 < nwork; p0 += C * kSelectWarps * 4) {
           int ja[4], jv[4];   // cbuf rows of the two members of each pair
+          int pj[4];          // pair index of each work item
 #pragma unroll
           for (int j = 0; j < 4; ++j) {
-            const int p = min(p0 + j, npairs - 1);
+            const int wi = min(p0 + j, nwork - 1);
+            const int p = TC ? plist[wi] : wi;
+            pj[j] = p;
             int u = 0, rem = p;
             while (rem >= nL - 1 - u) { rem -= nL - 1 - u; ++u; }
             ja[j] = lp_row[u];
@@ -954,8 +1033,8 @@ select_kernel(const __grid_constant__ SelectArgs a) {
 #pragma unroll
           for (int j = 0; j < 4; ++j) {
             const float d = butterfly_sum(acc[j]);
-            if (p0 + j < npairs && lane < C)
-              st_cluster_f32(map_shared(&pairbuf[par * kMaxPairs + p0 + j], lane), d);
+            if (p0 + j < nwork && lane < C)
+              st_cluster_f32(map_shared(&pairbuf[par * kMaxPairs + pj[j]], lane), d);
           }
         }
       }
