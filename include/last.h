@@ -170,6 +170,13 @@ last_status last_prune(const last_problem *p, const void *q, const void *k, cons
 last_status last_scores_noalloc(const last_problem *p, const void *q, const void *k,
                                 float *w_out, void *stream);
 
+/* Diagnostic (no counterpart in the paper): runs one device-side bounded wait that
+ * nothing completes, with a short iteration limit, so that the next last_poll on
+ * `ws` (at least 256 bytes) returns LAST_ERR_TIMEOUT.  It exercises the path every
+ * device wait of the library takes when a wait expires, without hanging or
+ * faulting the GPU. */
+last_status last_check_bounded_wait(void *ws, void *stream);
+
 /* Synchronises `stream`, then reports the device-side flags of the last call
  * that used `ws`: LAST_OK, LAST_ERR_DEVICE_INDEX, or LAST_ERR_TIMEOUT (a wait
  * on an asynchronous copy gave up after its iteration limit instead of hanging;

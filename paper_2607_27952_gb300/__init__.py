@@ -35,7 +35,7 @@ LAST_DTYPE_BF16 = 1
 EXPORTED = ("last_workspace_size", "last_scores", "last_select", "last_gather", "last_prune",
             "last_poll", "last_budget", "last_status_string", "last_error_message",
             "last_scores_noalloc", "last_select_topk", "last_scores_rows",
-            "last_scores_rows_workspace_size")
+            "last_scores_rows_workspace_size", "last_check_bounded_wait")
 
 
 class LastError(RuntimeError):
@@ -83,6 +83,7 @@ def load_library(path: str = LIB_PATH):
     lib.last_scores_rows_workspace_size.argtypes = [PP, PI, PI, ctypes.POINTER(ctypes.c_size_t)]
     lib.last_prune.argtypes = [PP, P, P, P, P, P, P, P, ctypes.c_size_t, P]
     lib.last_poll.argtypes = [P, P]
+    lib.last_check_bounded_wait.argtypes = [P, P]
     lib.last_scores_noalloc.argtypes = [PP, P, P, P, P]
     lib.last_budget.argtypes = [ctypes.c_int32, ctypes.c_int32, ctypes.c_int32]
     lib.last_budget.restype = ctypes.c_int32
@@ -92,7 +93,8 @@ def load_library(path: str = LIB_PATH):
     lib.last_error_message.restype = ctypes.c_char_p
     for name in ("last_workspace_size", "last_scores", "last_select", "last_gather",
                  "last_prune", "last_poll", "last_scores_noalloc", "last_select_topk",
-                 "last_scores_rows", "last_scores_rows_workspace_size"):
+                 "last_scores_rows", "last_scores_rows_workspace_size",
+                 "last_check_bounded_wait"):
         getattr(lib, name).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -244,6 +246,11 @@ def last_prune(problem: Problem, q, k, x, w_out, idx_out, x_out, ws, stream=None
     p, n = _ws(ws)
     _check(load_library().last_prune(problem.ref, _ptr(q), _ptr(k), _ptr(x), _ptr(w_out),
                                      _ptr(idx_out), _ptr(x_out), p, n, _stream(stream)))
+
+
+def last_check_bounded_wait(ws, stream=None):
+    p, _ = _ws(ws)
+    _check(load_library().last_check_bounded_wait(p, _stream(stream)))
 
 
 def last_poll(ws, stream=None):

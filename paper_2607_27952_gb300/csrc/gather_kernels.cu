@@ -53,3 +53,39 @@ cudaError_t launch_gather(const Plan &pl, const void *x, const int32_t *idx, voi
 }
 
 }  // namespace last
+
+// Diagnostic of the bounded-wait path: one thread waits on an mbarrier that nothing
+// completes, with a short iteration limit, and reports the expiry through the
+// workspace error word -- the same path every device wait of the library takes.
+namespace last {
+
+__global__ void bounded_wait_check_kernel(unsigned *err, uint32_t limit) {
+  __shared__ unsigned long long bar;
+  if (threadIdx.x != 0) return;
+  mbar_init(&bar, 1);   // expects one arrival that never comes
+  fence_mbar_init();
+  for (uint32_t i = 0; i < limit; ++i)
+    if (mbar_try_wait(&bar, 0)) return;
+  atomicOr(err, kErrTimeout);
+}
+
+}  // namespace last
+
+extern "C" last_status last_check_bounded_wait(void *ws, void *stream) {
+  using namespace last;
+  if (ws == nullptr) {
+    set_error("workspace is NULL");
+    return LAST_ERR_INVALID_ARG;
+  }
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaError_t e = cudaMemsetAsync(ws, 0, sizeof(unsigned), s);
+  if (e == cudaSuccess) {
+    bounded_wait_check_kernel<<<1, 32, 0, s>>>(static_cast<unsigned *>(ws), 1u << 12);
+    e = cudaGetLastError();
+  }
+  if (e != cudaSuccess) {
+    set_error(std::string("bounded-wait check: ") + cudaGetErrorString(e));
+    return LAST_ERR_CUDA;
+  }
+  return LAST_OK;
+}

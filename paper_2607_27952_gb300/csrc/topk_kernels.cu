@@ -2,7 +2,8 @@
 // highest importance score w~ per request, ties to the lower index, returned in
 // ascending index order (Eq. 12's sort(S)).
 //
-// topk_kernel: one CTA per request.  Every token gets the 64-bit key
+// topk_kernel: one CTA per request; a request of up to kTopkCacheTokens scores
+// keeps them in shared memory for every pass.  Every token gets the 64-bit key
 // (order-preserving bits of w~ << 32) | (0xffffffff - i), the same key the
 // greedy's argmax uses: keys are unique, larger key = kept first.  An MSB-first
 // radix select over 8-bit digits finds the k-th largest key T (stopping early
@@ -13,13 +14,17 @@
 #include "last_device.cuh"
 #include "last_internal.h"
 
+#include <algorithm>
+
 namespace last {
 
-constexpr int kTopkThreads = 512;
+constexpr int kTopkThreads = 1024;
+constexpr int kTopkCacheTokens = 48 * 1024;   // 192 KB of scores
 
 __global__ void __launch_bounds__(kTopkThreads)
 topk_kernel(const float *__restrict__ w, const int32_t *__restrict__ meta,
-            int32_t *__restrict__ idx_out) {
+            int32_t *__restrict__ idx_out, int cache_tokens) {
+  extern __shared__ float wcache[];
   constexpr int kWarps = kTopkThreads / 32;
   __shared__ unsigned hist[256];
   __shared__ unsigned long long s_prefix;
@@ -29,9 +34,15 @@ topk_kernel(const float *__restrict__ w, const int32_t *__restrict__ meta,
   const int32_t *m = meta + blockIdx.x * kMetaFields;
   const int N = m[kNumVis], k = m[kNumKeep];
   if (k <= 0) return;
-  const float *wb = w + m[kVisOff];
+  const float *wg = w + m[kVisOff];
   int32_t *out = idx_out + m[kKeepOff];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const bool cached = N <= cache_tokens;
+  if (cached) {
+    for (int i = tid; i < N; i += kTopkThreads) wcache[i] = wg[i];
+    __syncthreads();
+  }
+  const float *wb = cached ? wcache : wg;
 
   unsigned long long prefix = 0, mask = 0;
   unsigned need = static_cast<unsigned>(k);
@@ -47,8 +58,18 @@ topk_kernel(const float *__restrict__ w, const int32_t *__restrict__ meta,
           const unsigned long long key = argmax_key(wb[i], i);
           if ((key & mask) == prefix) digit = static_cast<unsigned>(key >> pos) & 255u;
         }
-        const unsigned peers = __match_any_sync(0xffffffffu, digit);
-        if (digit < 256u && lane == __ffs(peers) - 1) atomicAdd(&hist[digit], __popc(peers));
+        // common case: every counting lane of the warp has the same digit -> one add
+        const unsigned counting = __ballot_sync(0xffffffffu, digit < 256u);
+        const unsigned dmin = __reduce_min_sync(0xffffffffu, digit);
+        const unsigned dmax = __reduce_max_sync(0xffffffffu, digit < 256u ? digit : 0u);
+        if (counting == 0u) {
+          // nothing to count in this group of keys
+        } else if (dmin == dmax) {
+          if (lane == __ffs(counting) - 1) atomicAdd(&hist[dmin], __popc(counting));
+        } else {
+          const unsigned peers = __match_any_sync(0xffffffffu, digit);
+          if (digit < 256u && lane == __ffs(peers) - 1) atomicAdd(&hist[digit], __popc(peers));
+        }
       }
       __syncthreads();
       if (warp == 0) {
@@ -112,8 +133,20 @@ topk_kernel(const float *__restrict__ w, const int32_t *__restrict__ meta,
 cudaError_t launch_topk(const Plan &pl, const float *w, int32_t *idx_out, char *ws,
                         cudaStream_t s) {
   if (pl.total_keep == 0 || pl.B == 0) return cudaSuccess;
-  topk_kernel<<<pl.B, kTopkThreads, 0, s>>>(
-      w, reinterpret_cast<const int32_t *>(ws + pl.off_meta), idx_out);
+  int dev = 0, optin = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+  // cache every request's scores when they fit (the shared memory of the
+  // kernel's own arrays stays within the 48 KB static default)
+  const int cache = std::min<int>(std::min(kTopkCacheTokens, pl.max_vis),
+                                  std::max(0, (optin - 8 * 1024) / 4));
+  const size_t smem = sizeof(float) * (size_t)cache;
+  if (smem > 48 * 1024) {
+    cudaError_t e = cudaFuncSetAttribute(topk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+  }
+  topk_kernel<<<pl.B, kTopkThreads, smem, s>>>(
+      w, reinterpret_cast<const int32_t *>(ws + pl.off_meta), idx_out, cache);
   return cudaGetLastError();
 }
 
