@@ -5,7 +5,9 @@
 //   a pair share one row K[key][g][0..D): lane h of the pair reads the 16-byte
 //   segments h, h + 2, h + 4, ... so every warp-wide load fills whole 32-byte
 //   sectors, and forms partial logits of the G = Hq/Hkv q-heads of g in
-//   registers from the pre-scaled q held in shared memory (broadcast reads).
+//   registers from q held in shared memory (broadcast reads): bf16 q as stored,
+//   one mixed-precision fma.rn.f32.bf16 per element and the scale applied to the
+//   dot; fp32 q pre-scaled.
 //   One xor shuffle joins the pair.  The chunk's logits go to shared memory;
 //   per (layer, head) the CTA then writes the chunk's max and its sums of
 //   2^(z - max) over all keys and over the visual keys, and the visual logits.
@@ -48,10 +50,14 @@ template <typename T, int G>
 __global__ void __launch_bounds__(kScoreThreads, 3)
 score_logits_kernel(const ScoreArgs a) {
   constexpr int V = Elem<T>::kPerVec;   // elements per 16-byte segment
+  constexpr bool kBf16 = sizeof(T) == 2;
   extern __shared__ __align__(16) float smem_f[];
   const int Hq = a.Hq, D = a.D;
-  float *qs = smem_f;                   // [Hq][D] pre-scaled q
-  float *zbuf = smem_f + Hq * D;        // [chunk][Hq + 1] logits
+  // q of the item: bf16 as stored (one mixed-precision fma per element, the scale
+  // applied to the dot), fp32 pre-scaled
+  float *qs = smem_f;                   // [Hq][D] fp32, or bf16 in the first half
+  const unsigned char *qs_b = reinterpret_cast<const unsigned char *>(smem_f);
+  float *zbuf = smem_f + (kBf16 ? (Hq * D + 1) / 2 : Hq * D);   // [chunk][Hq + 1] logits
   const int ldz = Hq + 1;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int nseg = D / V;                 // segments per row
@@ -100,10 +106,14 @@ score_logits_kernel(const ScoreArgs a) {
     {
       const T *qb = static_cast<const T *>(a.q) + ((long long)b * a.L + l) * Hq * D;
       for (int v = tid; v < Hq * D / V; v += kScoreThreads) {
-        float e[V];
-        Elem<T>::widen(ldg(qb + v * V), e);
+        if constexpr (kBf16) {
+          reinterpret_cast<U4 *>(smem_f)[v] = ldg(qb + v * V);
+        } else {
+          float e[V];
+          Elem<T>::widen(ldg(qb + v * V), e);
 #pragma unroll
-        for (int x = 0; x < V; ++x) qs[v * V + x] = e[x] * a.qscale;
+          for (int x = 0; x < V; ++x) qs[v * V + x] = e[x] * a.qscale;
+        }
       }
     }
     __syncthreads();
@@ -113,6 +123,7 @@ score_logits_kernel(const ScoreArgs a) {
       int kk, g;
       const T *row = row_of(task, &ok, &kk, &g);
       const float *qg = qs + g * G * D;
+      const unsigned char *qgb = qs_b + (size_t)g * G * D * 2;
       float acc[G];
 #pragma unroll
       for (int gg = 0; gg < G; ++gg) acc[gg] = 0.f;
@@ -122,18 +133,32 @@ score_logits_kernel(const ScoreArgs a) {
         for (int j = 0; j < kSegBatch; ++j) {
           const int seg = 2 * (s0 + j) + half;
           if (seg < nseg) {
-            float e[V];
-            Elem<T>::widen(buf[j], e);
-            const float *qc = qg + seg * V;
+            if constexpr (kBf16) {
+              const uint32_t kw[4] = {buf[j].x, buf[j].y, buf[j].z, buf[j].w};
 #pragma unroll
-            for (int gg = 0; gg < G; ++gg) {
+              for (int gg = 0; gg < G; ++gg) {
+                const U4 qv = lds(qgb + ((size_t)gg * D + seg * V) * 2);
+                const uint32_t qw[4] = {qv.x, qv.y, qv.z, qv.w};
 #pragma unroll
-              for (int x = 0; x < V; x += 4) {
-                const float4 qv = *reinterpret_cast<const float4 *>(qc + gg * D + x);
-                acc[gg] = fmaf(qv.x, e[x], acc[gg]);
-                acc[gg] = fmaf(qv.y, e[x + 1], acc[gg]);
-                acc[gg] = fmaf(qv.z, e[x + 2], acc[gg]);
-                acc[gg] = fmaf(qv.w, e[x + 3], acc[gg]);
+                for (int hw = 0; hw < 4; ++hw) {
+                  acc[gg] = fma_bf16_lo(qw[hw], kw[hw], acc[gg]);
+                  acc[gg] = fma_bf16_hi(qw[hw], kw[hw], acc[gg]);
+                }
+              }
+            } else {
+              float e[V];
+              Elem<T>::widen(buf[j], e);
+              const float *qc = qg + seg * V;
+#pragma unroll
+              for (int gg = 0; gg < G; ++gg) {
+#pragma unroll
+                for (int x = 0; x < V; x += 4) {
+                  const float4 qv = *reinterpret_cast<const float4 *>(qc + gg * D + x);
+                  acc[gg] = fmaf(qv.x, e[x], acc[gg]);
+                  acc[gg] = fmaf(qv.y, e[x + 1], acc[gg]);
+                  acc[gg] = fmaf(qv.z, e[x + 2], acc[gg]);
+                  acc[gg] = fmaf(qv.w, e[x + 3], acc[gg]);
+                }
               }
             }
           }
@@ -142,8 +167,9 @@ score_logits_kernel(const ScoreArgs a) {
 #pragma unroll
       for (int gg = 0; gg < G; ++gg) acc[gg] += __shfl_xor_sync(0xffffffffu, acc[gg], 1);
       if (ok && half == 0) {
+        const float sc = kBf16 ? a.qscale : 1.0f;   // bf16: the scale goes on the dot
 #pragma unroll
-        for (int gg = 0; gg < G; ++gg) zbuf[kk * ldz + g * G + gg] = acc[gg];
+        for (int gg = 0; gg < G; ++gg) zbuf[kk * ldz + g * G + gg] = acc[gg] * sc;
       }
     }
     __syncthreads();

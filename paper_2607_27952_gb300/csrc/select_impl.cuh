@@ -61,6 +61,7 @@ constexpr int kTcBM = 128, kTcBK = 64;             // MMA M; K elements per 128-
 constexpr int kTcMaxStages = 12;                   // TMA ring depth (runtime a.tc_stages)
 constexpr int kTcBoxBytes = kTcBM * kTcBK * 2;     // one A box (128 rows x 64 elements): 16 KB
 constexpr int kTmemCols = 512;                     // TMEM columns per SM
+constexpr int kGramChains = 4;                     // accumulators of the list's Gram
 
 struct SelectArgs {
   CUtensorMap tmap;      // X as [total_vis][dv] bf16, box 64 x 128, 128-byte swizzle (tc only)
@@ -934,15 +935,18 @@ select_kernel(const __grid_constant__ SelectArgs a) {
           __syncthreads();
           tc_fence_after();
           const uint32_t gcol = (uint32_t)(((a.tpc_max + kTcBM - 1) / kTcBM) * lcap);
+          // K blocks alternate over kGramChains accumulators (independent MMA chains),
+          // added in the epilogue
           if (threadIdx.x == 32) {
             const uint32_t idesc = umma_idesc_bf16(kTcBM, lcap);
             const int nkb = tc_kblocks(dv);
             for (int kb = 0; kb < nkb; ++kb)
 #pragma unroll
               for (int k = 0; k < kTcBK / 16; ++k)
-                umma_bf16(tmem + gcol, umma_desc_sw128(cbuf_sa + kb * lcap * 128 + k * 32),
+                umma_bf16(tmem + gcol + (uint32_t)((kb % kGramChains) * lcap),
+                          umma_desc_sw128(cbuf_sa + kb * lcap * 128 + k * 32),
                           umma_desc_sw128(cbuf_sa + kb * lcap * 128 + k * 32), idesc,
-                          (kb | k) != 0 ? 1u : 0u);
+                          (kb >= kGramChains || k != 0) ? 1u : 0u);
             umma_commit(tpair);
           }
           __syncwarp();
@@ -950,12 +954,20 @@ select_kernel(const __grid_constant__ SelectArgs a) {
           tc_pph ^= 1u;
           tc_fence_after();
           if (warp == 0) {   // TMEM lanes 0..31 and the columns: cbuf rows
+            const int nch = min(kGramChains, tc_kblocks(dv));
             for (int v0 = 0; v0 < lcap; v0 += 16) {
-              uint32_t raw[16];
-              tmem_ld16(tmem + gcol + (uint32_t)v0, raw);
+              float sum[16];
+#pragma unroll
+              for (int j = 0; j < 16; ++j) sum[j] = 0.f;
+              for (int ch = 0; ch < nch; ++ch) {
+                uint32_t raw[16];
+                tmem_ld16(tmem + gcol + (uint32_t)(ch * lcap + v0), raw);
+#pragma unroll
+                for (int j = 0; j < 16; ++j) sum[j] += __uint_as_float(raw[j]);
+              }
 #pragma unroll
               for (int j = 0; j < 16; ++j)
-                if (lane < lcap) gram[lane * kLcap + v0 + j] = __uint_as_float(raw[j]);
+                if (lane < lcap) gram[lane * kLcap + v0 + j] = sum[j];
             }
           }
           tc_fence_before();

@@ -186,8 +186,10 @@ cudaError_t launch_select(const Plan &pl, const float *w, const void *x, int32_t
       // stages of kps boxes: the largest kps (<= 4) that still leaves 2 stages
       for (int lc = (c <= 4 ? kLcap : kLcap / 2); lc >= kLcap / 2 && lcap_c == 0; lc /= 2) {
         const size_t fixed = select_smem(0, rb, tpc_c, 0, tb_c, pl.elem, lc, 1, 0).total;
-        // TMEM: lc columns per tile plus lc for the list's Gram
-        if (fixed + 2 * (size_t)kTcBoxBytes > (size_t)di.optin || (tiles + 1) * lc > kTmemCols) continue;
+        // TMEM: lc columns per tile plus kGramChains x lc for the list's Gram
+        if (fixed + 2 * (size_t)kTcBoxBytes > (size_t)di.optin ||
+            (tiles + kGramChains) * lc > kTmemCols)
+          continue;
         const size_t room = di.optin - fixed;
         kps_c = 1;
         while (kps_c < 4 && room >= 2 * (size_t)(2 * kps_c) * kTcBoxBytes) kps_c *= 2;
@@ -265,7 +267,7 @@ cudaError_t launch_select(const Plan &pl, const float *w, const void *x, int32_t
   a.lcap = lcap;
   a.err = reinterpret_cast<unsigned *>(ws + pl.off_err);
   if (tc) {
-    const int cols = ((tpc + kTcBM - 1) / kTcBM + 1) * lcap;   // tiles + the list Gram
+    const int cols = ((tpc + kTcBM - 1) / kTcBM + kGramChains) * lcap;   // tiles + the list Gram
     uint32_t tcols = 32;
     while ((int)tcols < cols) tcols *= 2;
     a.tmem_cols = tcols;
