@@ -13,6 +13,14 @@
  *   3. last_gather  Eq. 12: the kept rows of X in ascending index order.
  *   last_prune runs 1-3 back to back on one stream.
  *
+ * Variants the paper evaluates beside the method:
+ *   last_select_topk  Table 5: keep the k_b highest scores (no diversity term).
+ *   last_scores_rows  Table 4: scores from the attention rows of several query
+ *                     positions (First, Middle, All Mean) instead of p* alone.
+ * Deployment aids without a counterpart in the paper: last_scores_noalloc
+ * (scoring without a caller workspace) and last_check_bounded_wait (exercises
+ * the reporting of an expired device wait).
+ *
  * Conventions shared by every entry point
  *   - All tensors are DEVICE pointers (caller-allocated, e.g. torch tensors);
  *     the library allocates no device memory.  Scratch lives in a caller
