@@ -218,11 +218,19 @@ last_status last_scores(const last_problem *p, const void *q, const void *k, flo
   return LAST_OK;
 }
 
+namespace {
+last_status check_select_fits(const last::Plan &pl) {
+  std::string why;
+  return last::select_fits(pl, &why) ? LAST_OK : fail(LAST_ERR_UNSUPPORTED, why);
+}
+}  // namespace
+
 last_status last_select(const last_problem *p, const float *w, const void *x, int32_t *idx_out,
                         void *x_out, void *ws, size_t ws_bytes, void *stream) {
   Plan pl;
   last_status st = make_plan(p, false, true, &pl);
   if (st != LAST_OK) return st;
+  if ((st = check_select_fits(pl)) != LAST_OK) return st;
   if ((st = check_ws(pl, ws, ws_bytes)) != LAST_OK) return st;
   if (pl.total_keep > 0 && (w == nullptr || x == nullptr || idx_out == nullptr))
     return fail(LAST_ERR_INVALID_ARG, "w, x and idx_out are required");
@@ -287,6 +295,7 @@ last_status last_prune(const last_problem *p, const void *q, const void *k, cons
   Plan pl;
   last_status st = make_plan(p, true, true, &pl);
   if (st != LAST_OK) return st;
+  if ((st = check_select_fits(pl)) != LAST_OK) return st;
   if ((st = check_ws(pl, ws, ws_bytes)) != LAST_OK) return st;
   if (pl.total_vis > 0 && (q == nullptr || k == nullptr || x == nullptr))
     return fail(LAST_ERR_INVALID_ARG, "q, k and x are required");

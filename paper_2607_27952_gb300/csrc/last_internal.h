@@ -75,5 +75,7 @@ int score_chunk_keys(int num_kv_heads);
 // Checks the compiled limits of the scoring / selection kernels.
 bool scores_supported(const Plan &pl, std::string *why);
 bool select_supported(const Plan &pl, std::string *why);
+// Whether the greedy selection's shared-memory plan holds the longest request.
+bool select_fits(const Plan &pl, std::string *why);
 
 }  // namespace last

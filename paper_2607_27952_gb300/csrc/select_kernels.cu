@@ -141,6 +141,19 @@ bool select_supported(const Plan &pl, std::string *why) {
   return true;
 }
 
+bool select_fits(const Plan &pl, std::string *why) {
+  // The largest request: the CUDA-core update's per-token state of one of 16
+  // clustered CTAs, with a row ring and no row cache, within sm_100-class shared
+  // memory (the launch itself takes the device's own figure).
+  const int tpc = (pl.max_vis + kMaxCluster - 1) / kMaxCluster;
+  const int tb = select_tb(pl.elem, false, tpc);
+  if (select_smem(0, pl.dv * pl.elem, tpc, 1, tb, pl.elem, kLcap / 2).total > (size_t)kSmemOptinSm100) {
+    if (why) *why = "a request has too many visual tokens for the selection's shared-memory plan";
+    return false;
+  }
+  return true;
+}
+
 // Bound on |d~ - d| between a tensor-core distance d~ = 1 - (dot~ r_i) r_j and the
 // canonical one, in units of cosine distance.  Both dots carry exact bf16 products;
 // the canonical order adds each lane's dv/256 * 8 products and five butterfly levels
@@ -167,15 +180,21 @@ cudaError_t launch_select(const Plan &pl, const float *w, const void *x, int32_t
   //   waves x (one round's update + round overhead)
   // (the round count of a request does not depend on C to first order); small
   // clusters raise the number of requests in flight, large ones shorten each round.
+  // When no cluster size fits the tensor-core update (its accumulators take a
+  // TMEM column per list entry and 128-row tile, so very long requests do not
+  // fit), the sizes are costed again for the CUDA-core update.
   int C = 0, tpc = 0, cache_rows = 0, ring = 0, lcap = kLcap / 2, stages = 0, kps = 1;
   size_t smem = 0;
   double best = 0.0;
   void *fn = nullptr;
+  for (int pass = 0; pass < 2 && C == 0; ++pass) {
+  if (pass == 1) {
+    if (!tc) break;
+    tc = false;
+  }
   for (int c = 1; c <= kMaxCluster; c = tc ? c + 1 : 2 * c) {
     const int tpc_c = (pl.max_vis + c - 1) / c;
-    // token block width of the kernel variant (the shared-memory plan depends on it):
-    // 2 for fp32 and the tensor-core update, else 4 unless a CTA owns few tokens
-    const int tb_c = (pl.elem == 4 || tc || tpc_c < 64) ? 2 : 4;
+    const int tb_c = select_tb(pl.elem, tc, tpc_c);
     void *fn_c = pick_select(pl.dtype, nch, tb_c, tc);
     int cache_c = 0, ring_c = 0, lcap_c = 0, stages_c = 0, kps_c = 1;
     size_t smem_c = 0;
@@ -241,6 +260,7 @@ cudaError_t launch_select(const Plan &pl, const float *w, const void *x, int32_t
       best = cost; C = c; tpc = tpc_c; cache_rows = cache_c; smem = smem_c; ring = ring_c;
       lcap = lcap_c; fn = fn_c; stages = stages_c; kps = kps_c;
     }
+  }
   }
   if (C == 0) return cudaErrorInvalidConfiguration;
   cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);

@@ -73,6 +73,10 @@ def test_scores_rejects_bad_problems_before_launch(lib, kw, status):
     (dict(feat_dim=100), last.LAST_ERR_INVALID_ARG),
     (dict(feat_dim=4096), last.LAST_ERR_UNSUPPORTED),
     (dict(cu_vis=[0, 6, 5]), last.LAST_ERR_INVALID_ARG),
+    (dict(dtype="f32", feat_dim=2048, cu_seqlens=[0, 10, 20020], cu_vis=[0, 6, 20006]),
+     last.LAST_ERR_UNSUPPORTED),                                             # N_b past smem
+    (dict(feat_dim=64, cu_seqlens=[0, 10, 140020], cu_vis=[0, 6, 140006]),
+     last.LAST_ERR_UNSUPPORTED),
 ])
 def test_select_rejects_bad_problems_before_launch(lib, kw, status):
     prob = _problem(**kw)
@@ -92,6 +96,18 @@ def test_topk_rejects_bad_arguments_before_launch(lib, kw, args, status):
     with pytest.raises(last.LastError) as e:
         last.last_select_topk(prob, 16, 16, (256, 1 << 30), stream=0, **args)
     assert e.value.status == status
+
+
+def test_long_requests_pass_topk_and_gather_validation(lib):
+    """The greedy's shared-memory bound on N_b applies to last_select alone: Top-k
+    and the gather take the same request up to their pointer checks."""
+    prob = _problem(dtype="f32", feat_dim=2048, cu_seqlens=[0, 10, 20020], cu_vis=[0, 6, 20006])
+    with pytest.raises(last.LastError) as e:
+        last.last_select_topk(prob, 16, 16, (256, 1 << 30), stream=0, x=24, x_out=16)
+    assert e.value.status == last.LAST_ERR_INVALID_ARG and "align" in str(e.value)
+    with pytest.raises(last.LastError) as e:
+        last.last_gather(prob, 24, 16, 16, (256, 1 << 30), stream=0)
+    assert e.value.status == last.LAST_ERR_INVALID_ARG and "align" in str(e.value)
 
 
 def test_topk_needs_no_sequence_fields(lib):
