@@ -62,7 +62,6 @@ constexpr int kTcMaxStages = 12;                   // TMA ring depth (runtime a.
 constexpr int kTcBoxBytes = kTcBM * kTcBK * 2;     // one A box (128 rows x 64 elements): 16 KB
 constexpr int kTmemCols = 512;                     // TMEM columns per SM
 constexpr int kGramChains = 4;                     // accumulators of the list's Gram
-constexpr int kSmemOptinSm100 = 232448;            // opt-in shared memory per CTA, sm_100 class
 
 struct SelectArgs {
   CUtensorMap tmap;      // X as [total_vis][dv] bf16, box 64 x 128, 128-byte swizzle (tc only)
@@ -97,11 +96,6 @@ __host__ __device__ inline size_t align16(size_t v) { return (v + 15) & ~size_t(
 // elem bytes) per lane.
 __host__ __device__ inline size_t ring_bytes(int ring, int tb, int elem) {
   return ring ? (size_t)kSelectWarps * kRing * tb * 8 * elem * 32 : 0;
-}
-// Token block width of the kernel variant (the shared-memory plan depends on it):
-// 2 for fp32 and the tensor-core update, else 4 unless a CTA owns few tokens.
-__host__ __device__ inline int select_tb(int elem, bool tc, int tpc_max) {
-  return (elem == 4 || tc || tpc_max < 64) ? 2 : 4;
 }
 __host__ __device__ inline int blocks_per_warp(int tpc_max, int tb) {
   return (tpc_max + kSelectWarps * tb - 1) / (kSelectWarps * tb);

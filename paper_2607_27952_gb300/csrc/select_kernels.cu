@@ -131,6 +131,14 @@ bool encode_x_map(CUtensorMap *m, const void *x, long long rows, int dv) {
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Opt-in shared memory per CTA of the sm_100 class, for checks made before a
+// device is at hand.
+constexpr int kSmemOptinSm100 = 232448;
+
+// Token block width of the kernel variant (the shared-memory plan depends on it):
+// 2 for fp32 and the tensor-core update, else 4 unless a CTA owns few tokens.
+int select_tb(int elem, bool tc, int tpc_max) { return (elem == 4 || tc || tpc_max < 64) ? 2 : 4; }
+
 }  // namespace
 
 bool select_supported(const Plan &pl, std::string *why) {
