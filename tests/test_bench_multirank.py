@@ -52,3 +52,21 @@ def test_reference_arm_runs_on_rank_zero_only(monkeypatch, capsys):
         gpus, steps, warmup, budget = 2, 1, 0, "mixed"
     bench.run_reference(A, rank=1, world=2)
     assert capsys.readouterr().out == ""
+
+
+def test_reference_arm_runs_one_request_per_host_thread(capsys):
+    """The oracle arm runs whole requests concurrently, one per host thread, and
+    reports those threads as its cores."""
+    import json
+    import bench
+
+    class A:
+        gpus, steps, warmup, budget, workload = 1, 1, 0, "mixed", "c1"
+        source, rows, selector = "last", 32, "greedy"
+    bench.run_reference(A, rank=0, world=1)
+    line = json.loads(capsys.readouterr().out.strip().splitlines()[-1])
+    threads = bench.host_threads()
+    assert line["impl"] == "reference" and line["cpu_baseline"]["cores"] == threads
+    assert line["value"] > 0 and line["e2e"]["h2d_bytes_per_step"] == 0
+    # visual tokens per step: one 576-token request per thread
+    assert abs(line["visual_tokens_scored_per_s"] / line["value"] - 576) < 1e-6
