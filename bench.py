@@ -319,16 +319,16 @@ def run_reference(args, rank, world):
     oracle.build()
     threads = host_threads()
 
-    def step(i):
-        ids = [(i * threads + j) % wl.batch for j in range(threads)]
-        return oracle_requests_parallel(oracle, wl, ids, threads, args.selector, rows)
+    def requests(first_step, nsteps):
+        return [(i * threads + j) % wl.batch
+                for i in range(first_step, first_step + nsteps) for j in range(threads)]
 
-    for i in range(args.warmup):
-        step(i)
+    # the steps' requests go through one pool without a barrier between steps, so
+    # that no core waits for a step's slowest request
+    oracle_requests_parallel(oracle, wl, requests(0, args.warmup), threads, args.selector, rows)
     t0 = time.perf_counter()
-    toks = 0
-    for i in range(args.steps):
-        toks += step(args.warmup + i)
+    toks = oracle_requests_parallel(oracle, wl, requests(args.warmup, args.steps), threads,
+                                    args.selector, rows)
     dt = time.perf_counter() - t0
     value = args.steps * threads / dt
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
@@ -341,7 +341,8 @@ def run_reference(args, rank, world):
             "visual_tokens_scored_per_s": toks / dt,
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle",
                              "sample": f"{threads} whole requests of the {args.workload} batch "
-                                       "per step, one per host thread, requests in turn"},
+                                       "per step, one per host thread, requests in turn, "
+                                       "steps not separated"},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
@@ -448,8 +449,11 @@ def main():
 
     e2e = None
     if not args.no_e2e:
-        e2e = measure_e2e(args, wl, prob, dev, stream, last, q, k, x,
-                          None if rows is None else (rows, rows_host[2], q_rows, ws_rows))
+        if rows is None and not topk:
+            e2e = measure_e2e_host(args, wl, prob, dev, last)
+        else:
+            e2e = measure_e2e(args, wl, prob, dev, stream, last, q, k, x,
+                              None if rows is None else (rows, rows_host[2], q_rows, ws_rows))
 
     comp, greedy = prune_bytes_moved(wl)
     sel_gbs = greedy / (select_ms / 1e3) / 1e9
@@ -513,10 +517,56 @@ def main():
         torch.distributed.destroy_process_group()
 
 
+def measure_e2e_host(args, wl, prob, dev, last):
+    """The same metric through the user call last_prune_host on pinned host buffers:
+    every step copies q, K and X to the device, prunes, and copies the kept indices and
+    rows back.  Steps alternate between two workspaces on two streams, as a server
+    would run them, so one step's copies overlap the previous step's kernels; the
+    timed region spans every step's copies and kernels."""
+    import torch
+    def pin(a):
+        if a.dtype == np.uint16:
+            return torch.from_numpy(a.view(np.int16)).view(torch.bfloat16).pin_memory()
+        return torch.from_numpy(a).pin_memory()
+    qh, kh, xh = pin(wl.q), pin(wl.k), pin(wl.x)
+    nkeep = int(wl.cu_keep[-1])
+    streams = [torch.cuda.Stream(dev), torch.cuda.Stream(dev)]
+    wss = [last.host_workspace(prob, dev) for _ in streams]
+    outs = [(torch.empty(nkeep, dtype=torch.int32).pin_memory(),
+             torch.empty((nkeep, wl.feat_dim), dtype=xh.dtype).pin_memory()) for _ in streams]
+
+    def step(i):
+        j = i % 2
+        last.last_prune_host(prob, qh, kh, xh, None, outs[j][0], outs[j][1], wss[j], streams[j])
+
+    for i in range(max(2, args.warmup // 2)):
+        step(i)
+    torch.cuda.synchronize(dev)
+    steps = max(4, args.steps // 2)
+    e0, e1, join = (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
+                    torch.cuda.Event())
+    e0.record(streams[0])
+    streams[1].wait_event(e0)
+    for i in range(steps):
+        step(i)
+    join.record(streams[1])
+    streams[0].wait_event(join)
+    e1.record(streams[0])
+    torch.cuda.synchronize(dev)
+    for ws in wss:
+        last.last_poll(ws, streams[0])
+    ms = e0.elapsed_time(e1)
+    h2d = int(qh.numel() + kh.numel() + xh.numel()) * xh.element_size()
+    d2h = int(outs[0][0].numel() * 4 + outs[0][1].numel() * outs[0][1].element_size())
+    return {"value": wl.batch * steps / (ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h, "steps": steps,
+            "call": "last_prune_host, pinned host buffers, two streams and workspaces alternating"}
+
+
 def measure_e2e(args, wl, prob, dev, stream, last, q_d, k_d, x_d, rows=None):
-    """The same metric through the user call last_prune with host buffers: each step
-    copies q, K, X from pinned host memory, prunes, and reads back the kept indices and
-    rows."""
+    """The same metric with host buffers for the variants: each step copies q (or the
+    query rows), K and X from pinned host memory, scores and selects through the
+    variant's calls, and reads back the kept indices and rows, on one stream."""
     import torch
     def pin(a):
         if a.dtype == np.uint16:
@@ -544,11 +594,9 @@ def measure_e2e(args, wl, prob, dev, stream, last, q_d, k_d, x_d, rows=None):
                 last.last_select_topk(prob, w_d, idx_d, ws, stream, x=x_d, x_out=xs_d)
             else:
                 last.last_select(prob, w_d, x_d, idx_d, ws, stream, x_out=xs_d)
-        elif args.selector == "topk":
+        else:
             last.last_scores(prob, q_d, k_d, w_d, ws, stream)
             last.last_select_topk(prob, w_d, idx_d, ws, stream, x=x_d, x_out=xs_d)
-        else:
-            last.last_prune(prob, q_d, k_d, x_d, None, idx_d, xs_d, ws, stream)
         idx_h.copy_(idx_d, non_blocking=True)
         xs_h.copy_(xs_d, non_blocking=True)
 

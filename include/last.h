@@ -17,13 +17,14 @@
  *   last_select_topk  Table 5: keep the k_b highest scores (no diversity term).
  *   last_scores_rows  Table 4: scores from the attention rows of several query
  *                     positions (First, Middle, All Mean) instead of p* alone.
- * Deployment aids without a counterpart in the paper: last_scores_noalloc
- * (scoring without a caller workspace) and last_check_bounded_wait (exercises
- * the reporting of an expired device wait).
+ * Deployment aids without a counterpart in the paper: last_prune_host (the
+ * whole path on host buffers, copies included), last_scores_noalloc (scoring
+ * without a caller workspace) and last_check_bounded_wait (exercises the
+ * reporting of an expired device wait).
  *
  * Conventions shared by every entry point
- *   - All tensors are DEVICE pointers (caller-allocated, e.g. torch tensors);
- *     the library allocates no device memory.  Scratch lives in a caller
+ *   - All tensors are DEVICE pointers (caller-allocated, e.g. torch tensors),
+ *     except those of last_prune_host; the library allocates no device memory.  Scratch lives in a caller
  *     workspace of at least last_workspace_size() bytes (256-byte aligned).
  *   - The offset arrays in last_problem are HOST arrays; each call validates
  *     them and copies a small plan into the workspace on `stream`.
@@ -167,6 +168,22 @@ last_status last_gather(const last_problem *p, const void *x, const int32_t *idx
 last_status last_prune(const last_problem *p, const void *q, const void *k, const void *x,
                        float *w_out, int32_t *idx_out, void *x_out,
                        void *ws, size_t ws_bytes, void *stream);
+
+/* last_prune on HOST buffers: q, k and x are read from host memory and idx_out,
+ * x_out (may be NULL) and w_out (may be NULL) are written to host memory, with
+ * the layouts above.  The call enqueues on `stream` the host-to-device copies of
+ * q, K and X into the device workspace, the whole path, and the device-to-host
+ * copies of the results, and returns; the host buffers must stay valid and
+ * unchanged until the stream has passed the call.  Pinned (page-locked) host
+ * memory keeps every copy asynchronous, so a caller alternating two workspaces
+ * on two streams overlaps one call's copies with another's kernels; pageable
+ * memory works but the copies then block the host.  The device workspace holds
+ * the plan and device copies of q, K, X, w~, the indices and the kept rows:
+ * last_host_workspace_size() bytes, 256-byte aligned. */
+last_status last_host_workspace_size(const last_problem *p, size_t *bytes);
+last_status last_prune_host(const last_problem *p, const void *q_host, const void *k_host,
+                            const void *x_host, float *w_out_host, int32_t *idx_out_host,
+                            void *x_out_host, void *ws, size_t ws_bytes, void *stream);
 
 /* last_scores without a caller workspace (the paper has no counterpart: this is
  * a deployment aid).  For callers that cannot allocate device memory at run time

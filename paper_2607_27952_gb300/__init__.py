@@ -35,7 +35,8 @@ LAST_DTYPE_BF16 = 1
 EXPORTED = ("last_workspace_size", "last_scores", "last_select", "last_gather", "last_prune",
             "last_poll", "last_budget", "last_status_string", "last_error_message",
             "last_scores_noalloc", "last_select_topk", "last_scores_rows",
-            "last_scores_rows_workspace_size", "last_check_bounded_wait")
+            "last_scores_rows_workspace_size", "last_check_bounded_wait",
+            "last_host_workspace_size", "last_prune_host")
 
 
 class LastError(RuntimeError):
@@ -82,6 +83,8 @@ def load_library(path: str = LIB_PATH):
     lib.last_scores_rows.argtypes = [PP, PI, PI, P, P, P, P, ctypes.c_size_t, P]
     lib.last_scores_rows_workspace_size.argtypes = [PP, PI, PI, ctypes.POINTER(ctypes.c_size_t)]
     lib.last_prune.argtypes = [PP, P, P, P, P, P, P, P, ctypes.c_size_t, P]
+    lib.last_host_workspace_size.argtypes = [PP, ctypes.POINTER(ctypes.c_size_t)]
+    lib.last_prune_host.argtypes = [PP, P, P, P, P, P, P, P, ctypes.c_size_t, P]
     lib.last_poll.argtypes = [P, P]
     lib.last_check_bounded_wait.argtypes = [P, P]
     lib.last_scores_noalloc.argtypes = [PP, P, P, P, P]
@@ -152,6 +155,24 @@ def _ptr(t) -> Optional[int]:
         raise ValueError("liblast takes device tensors")
     if not t.is_contiguous():
         raise ValueError("liblast takes contiguous tensors")
+    return t.data_ptr()
+
+
+def _host_ptr(t) -> Optional[int]:
+    """Address of a contiguous host buffer: a CPU torch tensor (pinned for
+    asynchronous copies) or a numpy array."""
+    if t is None:
+        return None
+    if isinstance(t, int):
+        return t
+    if isinstance(t, np.ndarray):
+        if not t.flags["C_CONTIGUOUS"]:
+            raise ValueError("host buffers must be contiguous")
+        return t.ctypes.data
+    if t.is_cuda:
+        raise ValueError("last_prune_host takes host buffers")
+    if not t.is_contiguous():
+        raise ValueError("host buffers must be contiguous")
     return t.data_ptr()
 
 
@@ -246,6 +267,29 @@ def last_prune(problem: Problem, q, k, x, w_out, idx_out, x_out, ws, stream=None
     p, n = _ws(ws)
     _check(load_library().last_prune(problem.ref, _ptr(q), _ptr(k), _ptr(x), _ptr(w_out),
                                      _ptr(idx_out), _ptr(x_out), p, n, _stream(stream)))
+
+
+def last_host_workspace_size(problem: Problem) -> int:
+    n = ctypes.c_size_t(0)
+    _check(load_library().last_host_workspace_size(problem.ref, ctypes.byref(n)))
+    return n.value
+
+
+def host_workspace(problem: Problem, device="cuda"):
+    """A torch uint8 device tensor of last_host_workspace_size bytes."""
+    import torch
+    return torch.empty(max(last_host_workspace_size(problem), 256), dtype=torch.uint8,
+                       device=device)
+
+
+def last_prune_host(problem: Problem, q, k, x, w_out, idx_out, x_out, ws, stream=None):
+    """last_prune on host buffers (pinned CPU tensors or numpy arrays); the copies
+    are enqueued on `stream` with the path, so the outputs are ready once the
+    stream has passed the call."""
+    p, n = _ws(ws)
+    _check(load_library().last_prune_host(problem.ref, _host_ptr(q), _host_ptr(k), _host_ptr(x),
+                                          _host_ptr(w_out), _host_ptr(idx_out),
+                                          _host_ptr(x_out), p, n, _stream(stream)))
 
 
 def last_check_bounded_wait(ws, stream=None):

@@ -178,6 +178,32 @@ last_status cuda_fail(cudaError_t e, const char *what) {
   return fail(LAST_ERR_CUDA, std::string(what) + ": " + cudaGetErrorString(e));
 }
 
+// Device copies of last_prune_host's tensors after the plan workspace, each
+// 256-byte aligned.
+struct HostLayout {
+  size_t q, k, x, w, idx, xo, total;
+  size_t q_bytes, k_bytes, x_bytes, w_bytes, idx_bytes, xo_bytes;
+};
+HostLayout host_layout(const Plan &pl) {
+  auto al = [](size_t v) { return (v + kAlign - 1) & ~(size_t)(kAlign - 1); };
+  HostLayout h;
+  h.q_bytes = (size_t)pl.B * pl.L * pl.Hq * pl.D * pl.elem;
+  h.k_bytes = (size_t)pl.L * pl.total_keys * pl.Hkv * pl.D * pl.elem;
+  h.x_bytes = (size_t)pl.total_vis * pl.dv * pl.elem;
+  h.w_bytes = (size_t)pl.total_vis * sizeof(float);
+  h.idx_bytes = (size_t)pl.total_keep * sizeof(int32_t);
+  h.xo_bytes = (size_t)pl.total_keep * pl.dv * pl.elem;
+  size_t o = al(pl.total_bytes);
+  h.q = o; o += al(h.q_bytes);
+  h.k = o; o += al(h.k_bytes);
+  h.x = o; o += al(h.x_bytes);
+  h.w = o; o += al(h.w_bytes);
+  h.idx = o; o += al(h.idx_bytes);
+  h.xo = o; o += al(h.xo_bytes);
+  h.total = o;
+  return h;
+}
+
 last_status stage(const Plan &pl, void *ws, cudaStream_t s) {
   cudaError_t e = cudaMemcpyAsync(ws, pl.host_blob.data(), pl.blob_bytes, cudaMemcpyHostToDevice, s);
   if (e != cudaSuccess) return cuda_fail(e, "plan copy");
@@ -311,6 +337,59 @@ last_status last_prune(const last_problem *p, const void *q, const void *k, cons
   if (e != cudaSuccess) return cuda_fail(e, "scoring launch");
   e = launch_select(pl, w, x, idx_out, x_out, wsc, s);
   if (e != cudaSuccess) return cuda_fail(e, "selection launch");
+  return LAST_OK;
+}
+
+last_status last_host_workspace_size(const last_problem *p, size_t *bytes) {
+  if (bytes == nullptr) return fail(LAST_ERR_INVALID_ARG, "bytes is NULL");
+  Plan pl;
+  last_status st = make_plan(p, true, true, &pl);
+  if (st != LAST_OK) return st;
+  *bytes = host_layout(pl).total;
+  return LAST_OK;
+}
+
+last_status last_prune_host(const last_problem *p, const void *q, const void *k, const void *x,
+                            float *w_out, int32_t *idx_out, void *x_out, void *ws, size_t ws_bytes,
+                            void *stream) {
+  Plan pl;
+  last_status st = make_plan(p, true, true, &pl);
+  if (st != LAST_OK) return st;
+  if ((st = check_select_fits(pl)) != LAST_OK) return st;
+  const HostLayout h = host_layout(pl);
+  if (ws == nullptr) return fail(LAST_ERR_INVALID_ARG, "workspace is NULL");
+  if ((reinterpret_cast<uintptr_t>(ws) & (kAlign - 1)) != 0)
+    return fail(LAST_ERR_INVALID_ARG, "workspace must be 256-byte aligned");
+  if (ws_bytes < h.total)
+    return fail(LAST_ERR_WORKSPACE_TOO_SMALL,
+                "last_prune_host's workspace needs " + std::to_string(h.total) + " bytes");
+  if (pl.total_vis > 0 && (q == nullptr || k == nullptr || x == nullptr))
+    return fail(LAST_ERR_INVALID_ARG, "q, k and x are required");
+  if (pl.total_keep > 0 && idx_out == nullptr)
+    return fail(LAST_ERR_INVALID_ARG, "idx_out is required");
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  char *wsc = static_cast<char *>(ws);
+  void *qd = wsc + h.q, *kd = wsc + h.k, *xd = wsc + h.x, *xod = wsc + h.xo;
+  float *wd = reinterpret_cast<float *>(wsc + h.w);
+  int32_t *idd = reinterpret_cast<int32_t *>(wsc + h.idx);
+  cudaError_t e = cudaSuccess;
+  // one copy per tensor
+  if (h.q_bytes && e == cudaSuccess) e = cudaMemcpyAsync(qd, q, h.q_bytes, cudaMemcpyHostToDevice, s);
+  if (h.k_bytes && e == cudaSuccess) e = cudaMemcpyAsync(kd, k, h.k_bytes, cudaMemcpyHostToDevice, s);
+  if (h.x_bytes && e == cudaSuccess) e = cudaMemcpyAsync(xd, x, h.x_bytes, cudaMemcpyHostToDevice, s);
+  if (e != cudaSuccess) return cuda_fail(e, "host-to-device copy");
+  if ((st = stage(pl, ws, s)) != LAST_OK) return st;
+  e = launch_scores(pl, qd, kd, wd, wsc, s);
+  if (e != cudaSuccess) return cuda_fail(e, "scoring launch");
+  e = launch_select(pl, wd, xd, idd, x_out != nullptr ? xod : nullptr, wsc, s);
+  if (e != cudaSuccess) return cuda_fail(e, "selection launch");
+  if (h.idx_bytes && e == cudaSuccess)
+    e = cudaMemcpyAsync(idx_out, idd, h.idx_bytes, cudaMemcpyDeviceToHost, s);
+  if (x_out != nullptr && h.xo_bytes && e == cudaSuccess)
+    e = cudaMemcpyAsync(x_out, xod, h.xo_bytes, cudaMemcpyDeviceToHost, s);
+  if (w_out != nullptr && h.w_bytes && e == cudaSuccess)
+    e = cudaMemcpyAsync(w_out, wd, h.w_bytes, cudaMemcpyDeviceToHost, s);
+  if (e != cudaSuccess) return cuda_fail(e, "device-to-host copy");
   return LAST_OK;
 }
 

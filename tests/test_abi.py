@@ -110,6 +110,30 @@ def test_long_requests_pass_topk_and_gather_validation(lib):
     assert e.value.status == last.LAST_ERR_INVALID_ARG and "align" in str(e.value)
 
 
+def test_host_workspace_holds_the_device_copies(lib):
+    prob = _problem()
+    n_ws = last.last_workspace_size(prob)
+    n_host = last.last_host_workspace_size(prob)
+    # q [2][1][4][64], K [1][30][2][64], X [14][256] bf16; w [14], idx [5], rows [5][256]
+    payload = (2 * 4 * 64 + 30 * 2 * 64 + 14 * 256) * 2 + 14 * 4 + 5 * 4 + 5 * 256 * 2
+    assert n_host >= n_ws + payload and n_host % 256 == 0
+
+
+@pytest.mark.parametrize("args,status", [
+    (dict(ws=(256, 1024)), last.LAST_ERR_WORKSPACE_TOO_SMALL),
+    (dict(ws=(300, 1 << 30)), last.LAST_ERR_INVALID_ARG),          # not 256-byte aligned
+    (dict(ws=(256, 1 << 30), idx_out=None), last.LAST_ERR_INVALID_ARG),
+    (dict(ws=(256, 1 << 30), k=None), last.LAST_ERR_INVALID_ARG),
+])
+def test_prune_host_rejects_bad_arguments_before_any_copy(lib, args, status):
+    call = dict(q=16, k=16, x=16, w_out=None, idx_out=16, x_out=None)
+    call.update(args)
+    ws = call.pop("ws")
+    with pytest.raises(last.LastError) as e:
+        last.last_prune_host(_problem(), ws=ws, stream=0, **call)
+    assert e.value.status == status
+
+
 def test_topk_needs_no_sequence_fields(lib):
     # scores-only fields may be absent; validation then fails only on the workspace
     prob = last.Problem(batch=1, num_layers=0, num_q_heads=0, num_kv_heads=0, head_dim=0,
