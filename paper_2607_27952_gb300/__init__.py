@@ -1,14 +1,15 @@
 """Python binding of liblast (GB300 / sm_103a) -- argument marshalling only.
 
 Every step of the path runs in the CUDA kernels of liblast.so; this module
-only turns torch tensors into device pointers and host offset arrays into the
-C problem struct.  There is no CPU fallback: if the library is missing, every
-call raises.
+only turns torch tensors (and, for last_prune_host, host buffers) into pointers
+and host offset arrays into the C problem struct.  There is no CPU fallback: if
+the library is missing, every call raises.
 
 Functions carry the names of the C entry points in include/last.h:
   last_workspace_size, last_scores, last_select, last_select_topk, last_gather,
-  last_prune, last_scores_noalloc, last_poll, last_budget, last_status_string,
-  last_error_message.
+  last_prune, last_host_workspace_size, last_prune_host, last_scores_rows,
+  last_scores_rows_workspace_size, last_scores_noalloc, last_check_bounded_wait,
+  last_poll, last_budget, last_status_string, last_error_message.
 """
 from __future__ import annotations
 
