@@ -148,7 +148,10 @@ last_status last_select_topk(const last_problem *p, const float *w, const void *
  * [head_dim] holds one query vector per row, layer and q-head; k as for
  * last_scores.  w_out [cu_vis[batch]] receives the visual probabilities summed
  * over rows, layers and q-heads and normalised per request (a mean over the rows
- * gives the same w~).  Limits: bf16 only; head_dim 64, 128, 192 or 256; rows x
+ * gives the same w~).  With one row per request (First, Middle, Last) the row
+ * at position pos is the last-row computation on keys 0 .. pos, and the call
+ * runs last_scores' kernels on the requests cut there (when G <= 8).
+ * Limits: bf16 only; head_dim 64, 128, 192 or 256; rows x
  * (num_q_heads / num_kv_heads) <= 256 and rows x layers x q-heads <= 6144 per
  * request.  The workspace is sized by last_scores_rows_workspace_size. */
 last_status last_scores_rows_workspace_size(const last_problem *p, const int32_t *cu_rows,

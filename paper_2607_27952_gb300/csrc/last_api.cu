@@ -26,7 +26,8 @@ bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 
 void set_error(const std::string &msg) { g_error = msg; }
 
-last_status make_plan(const last_problem *p, bool need_scores, bool need_select, Plan *pl) {
+last_status make_plan(const last_problem *p, bool need_scores, bool need_select, Plan *pl,
+                      const int32_t *seq_len) {
   if (p == nullptr) return fail(LAST_ERR_INVALID_ARG, "problem is NULL");
   if (p->batch < 0) return fail(LAST_ERR_INVALID_ARG, "batch < 0");
   if (p->dtype != LAST_DTYPE_F32 && p->dtype != LAST_DTYPE_BF16)
@@ -83,8 +84,11 @@ last_status make_plan(const last_problem *p, bool need_scores, bool need_select,
     pl->scale = p->softmax_scale > 0.f ? p->softmax_scale
                                        : (float)(1.0 / std::sqrt((double)p->head_dim));
     for (int b = 0; b < B; ++b) {
-      const int P = p->cu_seqlens[b + 1] - p->cu_seqlens[b];
+      const int P_full = p->cu_seqlens[b + 1] - p->cu_seqlens[b];
+      const int P = seq_len != nullptr ? seq_len[b] : P_full;
       const int n = p->cu_vis[b + 1] - p->cu_vis[b];
+      if (P > P_full)
+        return fail(LAST_ERR_INVALID_ARG, "request " + std::to_string(b) + ": cut beyond P_b");
       if (P < 1)
         return fail(LAST_ERR_INVALID_ARG, "request " + std::to_string(b) +
                                               ": P_b must be >= 1 (the query position)");
@@ -139,7 +143,7 @@ last_status make_plan(const last_problem *p, bool need_scores, bool need_select,
     m[kNumKeep] = p->cu_keep[b + 1] - p->cu_keep[b];
     if (have_seq && p->num_layers > 0) {
       m[kSeqStart] = p->cu_seqlens[b];
-      m[kSeqLen] = p->cu_seqlens[b + 1] - p->cu_seqlens[b];
+      m[kSeqLen] = seq_len != nullptr ? seq_len[b] : p->cu_seqlens[b + 1] - p->cu_seqlens[b];
       m[kVisStart] = p->vis_start[b];
       m[kChunkBase] = chunk;
       const int nch = (m[kSeqLen] + pl->chunk - 1) / pl->chunk;

@@ -55,7 +55,10 @@ struct Plan {
 
 // Validation + layout.  `need_scores` / `need_select` widen the checks to the
 // parts a call uses.  Returns LAST_OK or an error with a message set.
-last_status make_plan(const last_problem *p, bool need_scores, bool need_select, Plan *plan);
+// seq_len (nullable): per-request key counts P'_b <= P_b to score instead of P_b
+// (keys 0 .. P'_b - 1 of each request, whose last one is then the query row).
+last_status make_plan(const last_problem *p, bool need_scores, bool need_select, Plan *plan,
+                      const int32_t *seq_len = nullptr);
 
 void set_error(const std::string &msg);
 

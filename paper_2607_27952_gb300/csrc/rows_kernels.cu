@@ -439,6 +439,20 @@ size_t tmem_safe_smem(size_t operands, uint32_t cols) {
   return std::max(operands, per_sm / (512 / cols + 1) + 1);
 }
 
+// One query row per request: the row at position pos attends keys 0 .. pos, which
+// is the last-row computation of Eq. 6-8 on the request cut after pos, so the
+// last-row scoring kernels take it (the last_scores plan with P'_b = pos + 1).
+// Returns LAST_OK only when that plan applies.
+last_status single_row_plan(const last_problem *p, const int32_t *cu_rows, const int32_t *row_pos,
+                            Plan *lp) {
+  if (p->batch < 1 || cu_rows[p->batch] != p->batch) return LAST_ERR_UNSUPPORTED;
+  std::vector<int32_t> len(p->batch);
+  for (int b = 0; b < p->batch; ++b) len[b] = row_pos[b] + 1;
+  last_problem pc = *p;
+  if (pc.cu_keep == nullptr) pc.cu_keep = pc.cu_vis;   // scoring needs no budgets
+  return make_plan(&pc, true, false, lp, len.data());
+}
+
 }  // namespace
 }  // namespace last
 
@@ -450,7 +464,9 @@ extern "C" last_status last_scores_rows_workspace_size(const last_problem *p, co
   RowsPlan pl;
   last_status st = make_rows_plan(p, cu_rows, row_pos, &pl);
   if (st != LAST_OK) return st;
+  Plan lp;
   *bytes = pl.total_bytes;
+  if (single_row_plan(p, cu_rows, row_pos, &lp) == LAST_OK) *bytes = std::max(*bytes, lp.total_bytes);
   return LAST_OK;
 }
 
@@ -460,18 +476,27 @@ extern "C" last_status last_scores_rows(const last_problem *p, const int32_t *cu
   RowsPlan pl;
   last_status st = make_rows_plan(p, cu_rows, row_pos, &pl);
   if (st != LAST_OK) return st;
+  Plan lp;
+  const bool single = single_row_plan(p, cu_rows, row_pos, &lp) == LAST_OK;
+  const size_t need = single ? std::max(pl.total_bytes, lp.total_bytes) : pl.total_bytes;
   if (ws == nullptr) return rows_fail(LAST_ERR_INVALID_ARG, "workspace is NULL");
   if ((reinterpret_cast<uintptr_t>(ws) & (kAlignR - 1)) != 0)
     return rows_fail(LAST_ERR_INVALID_ARG, "workspace must be 256-byte aligned");
-  if (ws_bytes < pl.total_bytes)
-    return rows_fail(LAST_ERR_WORKSPACE_TOO_SMALL,
-                     "workspace needs " + std::to_string(pl.total_bytes) + " bytes");
+  if (ws_bytes < need)
+    return rows_fail(LAST_ERR_WORKSPACE_TOO_SMALL, "workspace needs " + std::to_string(need) + " bytes");
   if (pl.total_vis > 0 && (q_rows == nullptr || k == nullptr || w_out == nullptr))
     return rows_fail(LAST_ERR_INVALID_ARG, "q_rows, k and w_out are required");
   if ((reinterpret_cast<uintptr_t>(q_rows) & 15u) || (reinterpret_cast<uintptr_t>(k) & 15u))
     return rows_fail(LAST_ERR_INVALID_ARG, "q_rows and k must be 16-byte aligned");
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   char *wsc = static_cast<char *>(ws);
+  if (single) {
+    cudaError_t e = cudaMemcpyAsync(wsc, lp.host_blob.data(), lp.blob_bytes, cudaMemcpyHostToDevice, s);
+    if (e == cudaSuccess) e = launch_scores(lp, q_rows, k, w_out, wsc, s);
+    if (e != cudaSuccess) return rows_fail(LAST_ERR_CUDA, std::string("single-row scoring: ") +
+                                                            cudaGetErrorString(e));
+    return LAST_OK;
+  }
   cudaError_t e = cudaMemcpyAsync(wsc, pl.blob.data(), pl.blob_bytes, cudaMemcpyHostToDevice, s);
   if (e != cudaSuccess) return rows_fail(LAST_ERR_CUDA, std::string("plan copy: ") + cudaGetErrorString(e));
   if (pl.total_vis == 0 || pl.B == 0) return LAST_OK;

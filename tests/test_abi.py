@@ -166,6 +166,8 @@ def test_scores_rows_workspace_grows_with_rows(lib):
     one = last.last_scores_rows_workspace_size(prob, last.QueryRows([0, 1, 2], [9, 19]))
     many = last.last_scores_rows_workspace_size(prob, last.QueryRows([0, 3, 6], [6, 7, 9, 10, 15, 19]))
     assert many > one > 0
+    # one row per request runs the last-row kernels: the workspace holds their plan
+    assert one >= last.last_workspace_size(prob)
 
 
 def test_workspace_checks(lib):

@@ -70,3 +70,15 @@ def test_reference_arm_runs_one_request_per_host_thread(capsys):
     assert line["value"] > 0 and line["e2e"]["h2d_bytes_per_step"] == 0
     # visual tokens per step: one 576-token request per thread
     assert abs(line["visual_tokens_scored_per_s"] / line["value"] - 576) < 1e-6
+
+
+def test_scoring_kernel_count_per_source():
+    """gpu_launches counts the scoring kernels of each attention source: two for
+    the last row and for one row per request (G <= 8), four for several rows."""
+    import bench
+    from workloads import config, query_rows
+    wl = config("c2", batch=3, budget="mixed")
+    assert bench.scoring_kernels(wl) == 2
+    assert bench.scoring_kernels(wl, query_rows(wl, "first")[0]) == 2
+    assert bench.scoring_kernels(wl, query_rows(wl, "middle")[0]) == 2
+    assert bench.scoring_kernels(wl, query_rows(wl, "all", m_rows=8)[0]) == 4

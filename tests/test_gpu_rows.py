@@ -76,15 +76,26 @@ def test_rows_match_oracle(name, source):
 
 
 def test_last_row_equals_single_row_scoring():
-    """The Last source is the method's own Eq. 6-8: it agrees with last_scores."""
-    import torch
-    import paper_2607_27952_gb300 as last
+    """The Last source is the method's own Eq. 6-8: one row per request runs the
+    last-row scoring kernels (cut after the row), so it equals last_scores bit for
+    bit."""
     from gpu_util import DeviceWorkload
     wl = CASES["c3"]()
     cu, pos, q = make_rows(wl, "last", np.random.default_rng(8))
     w_rows = check(wl, cu, pos, q)
     w_one = DeviceWorkload(wl).scores()
-    np.testing.assert_allclose(w_rows, w_one, rtol=2e-3, atol=1e-30)
+    assert np.array_equal(w_rows.view(np.uint32), w_one.view(np.uint32))
+
+
+def test_single_row_beyond_the_last_row_kernels():
+    """G = 16 q-heads per kv-head is past the last-row kernels (G <= 8): one row per
+    request then runs on the multi-row kernels, still within tolerance."""
+    wl = custom(name="g16", seed=64, batch=3, n_vis=[120, 40, 260], n_text=[30, 5, 64],
+                num_layers=1, num_q_heads=32, num_kv_heads=2, head_dim=64, feat_dim=64,
+                dtype="bf16")
+    for source in ("first", "middle"):
+        cu, pos, q = make_rows(wl, source, np.random.default_rng(10))
+        check(wl, cu, pos, q)
 
 
 def test_many_rows_full_width():
