@@ -102,10 +102,12 @@ def test_prune_end_to_end(name):
 
 
 def test_prune_is_deterministic():
+    """Ten runs, bitwise-equal scores, indices and rows: every reduction has a fixed
+    order, and the only atomics fill a work list whose order no result depends on."""
     wl = MINI["c4"]()
     dw = DeviceWorkload(wl)
     a = dw.prune()
-    for _ in range(3):
+    for _ in range(9):
         b = dw.prune()
         for u, v in zip(a, b):
             assert np.array_equal(u.view(np.uint8), v.view(np.uint8))
