@@ -110,7 +110,9 @@ typedef struct {
   const int32_t *cu_keep;    /* [batch+1] */
 } last_problem;
 
-/* Bytes of device workspace every entry point below needs for `p`.
+/* Bytes of device workspace the entry points below need for `p`, except
+ * last_scores_rows and last_prune_host, which are sized by
+ * last_scores_rows_workspace_size and last_host_workspace_size.
  * Returns LAST_ERR_INVALID_ARG / LAST_ERR_UNSUPPORTED for a bad problem. */
 last_status last_workspace_size(const last_problem *p, size_t *bytes);
 
