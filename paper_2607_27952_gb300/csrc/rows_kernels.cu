@@ -450,7 +450,12 @@ last_status single_row_plan(const last_problem *p, const int32_t *cu_rows, const
   for (int b = 0; b < p->batch; ++b) len[b] = row_pos[b] + 1;
   last_problem pc = *p;
   if (pc.cu_keep == nullptr) pc.cu_keep = pc.cu_vis;   // scoring needs no budgets
-  return make_plan(&pc, true, false, lp, len.data());
+  // a probe: when the plan does not apply, the multi-row kernels run instead and the
+  // call's error message must not report the probe's rejection
+  const std::string saved = get_error();
+  const last_status st = make_plan(&pc, true, false, lp, len.data());
+  if (st != LAST_OK) set_error(saved);
+  return st;
 }
 
 }  // namespace
@@ -466,7 +471,7 @@ extern "C" last_status last_scores_rows_workspace_size(const last_problem *p, co
   if (st != LAST_OK) return st;
   Plan lp;
   *bytes = pl.total_bytes;
-  if (single_row_plan(p, cu_rows, row_pos, &lp) == LAST_OK) *bytes = std::max(*bytes, lp.total_bytes);
+  if (single_row_plan(p, cu_rows, row_pos, &lp) == LAST_OK) *bytes = std::max(*bytes, lp.score_bytes);
   return LAST_OK;
 }
 
@@ -478,7 +483,7 @@ extern "C" last_status last_scores_rows(const last_problem *p, const int32_t *cu
   if (st != LAST_OK) return st;
   Plan lp;
   const bool single = single_row_plan(p, cu_rows, row_pos, &lp) == LAST_OK;
-  const size_t need = single ? std::max(pl.total_bytes, lp.total_bytes) : pl.total_bytes;
+  const size_t need = single ? std::max(pl.total_bytes, lp.score_bytes) : pl.total_bytes;
   if (ws == nullptr) return rows_fail(LAST_ERR_INVALID_ARG, "workspace is NULL");
   if ((reinterpret_cast<uintptr_t>(ws) & (kAlignR - 1)) != 0)
     return rows_fail(LAST_ERR_INVALID_ARG, "workspace must be 256-byte aligned");

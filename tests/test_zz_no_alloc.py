@@ -3,8 +3,9 @@
 It serves callers that cannot allocate device memory at run time (for example a
 service that reserves all of its device memory at start-up).  Its scratch is a
 fixed array inside the library, so this test checks that two calls in a row give
-the same scores as last_scores with a caller workspace, within the score
-tolerance of the parity tests, and that an oversized problem is rejected.
+the oracle's scores and those of last_scores with a caller workspace, within the
+score tolerance of the parity tests, on problems of alternating size and dtype,
+and that an oversized problem is rejected.
 This file is collected last so that a stop-at-first-failure run has already run
 every other test.
 """
@@ -42,16 +43,25 @@ def _dev(a, dev):
 
 
 def test_noalloc_scores_match_workspace_path_twice(lib):
+    """Large, small, large again (bf16, GQA, fp32 in between): every call must ignore
+    the statistics and logits a previous, differently sized call left in the shared
+    scratch.  Each call is checked against the fp64 oracle (rtol 1e-3, the parity
+    tolerance) and against last_scores with a workspace, two calls in a row."""
     import torch
+    import oracle
     from workloads import config, custom
+    oracle.build()
     dev = torch.device("cuda:0")
-    cases = [config("c2", batch=6, budget="mixed"),
-             custom(name="gqa7", seed=5, batch=3, n_vis=[120, 33, 300], n_text=[7, 2, 19],
-                    n_before=[4, 0, 9], num_layers=2, num_q_heads=14, num_kv_heads=2,
-                    head_dim=64, feat_dim=64, dtype="bf16", keep=[8, 3, 30])]
-    for wl in cases:
+    large = config("c2", batch=6, budget="mixed")
+    small = custom(name="gqa7", seed=5, batch=3, n_vis=[120, 33, 300], n_text=[7, 2, 19],
+                   n_before=[4, 0, 9], num_layers=2, num_q_heads=14, num_kv_heads=2,
+                   head_dim=64, feat_dim=64, dtype="bf16", keep=[8, 3, 30])
+    fp32 = config("c1")
+    for wl in (large, small, fp32, large, small):
         prob = _problem(lib, wl)
         q, k = _dev(wl.q, dev), _dev(wl.k, dev)
+        want = oracle.scores(wl.q, wl.k, wl.cu_seqlens, wl.vis_start, wl.cu_vis,
+                             num_kv_heads=wl.num_kv_heads, scale=wl.scale)
         ref = torch.full((prob.total_vis,), float("nan"), device=dev)
         ws = lib.workspace(prob, dev)
         lib.last_scores(prob, q, k, ref, ws)
@@ -63,7 +73,8 @@ def test_noalloc_scores_match_workspace_path_twice(lib):
             torch.cuda.synchronize()
             got = out.cpu().numpy().astype(np.float64)
             assert np.isfinite(got).all()
-            assert np.allclose(got, ref, rtol=1e-3, atol=1e-30)
+            assert np.allclose(got, want, rtol=1e-3, atol=1e-30), wl.name
+            assert np.allclose(got, ref, rtol=1e-3, atol=1e-30), wl.name
 
 
 def test_noalloc_rejects_oversized_problem(lib):
