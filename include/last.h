@@ -164,7 +164,9 @@ last_status last_scores_rows(const last_problem *p, const int32_t *cu_rows,
 
 /* Eq. 12.  x_out[r] = x[cu_vis[b] + idx[r]] for r in request b's output range.
  * An index outside [0, N_b) leaves its row unwritten and makes last_poll
- * return LAST_ERR_DEVICE_INDEX. */
+ * return LAST_ERR_DEVICE_INDEX.  Any feat_dim that is a positive multiple of 8
+ * is accepted (the selection's own feat_dim <= 2048 limit does not apply); the
+ * workspace carries the plan and the device error word. */
 last_status last_gather(const last_problem *p, const void *x, const int32_t *idx,
                         void *x_out, void *ws, size_t ws_bytes, void *stream);
 

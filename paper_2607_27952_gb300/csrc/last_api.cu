@@ -25,6 +25,7 @@ bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 }  // namespace
 
 void set_error(const std::string &msg) { g_error = msg; }
+std::string get_error() { return g_error; }
 
 last_status make_plan(const last_problem *p, bool need_scores, bool need_select, Plan *pl,
                       const int32_t *seq_len) {
@@ -126,6 +127,22 @@ last_status make_plan(const last_problem *p, bool need_scores, bool need_select,
                        (size_t)pl->total_vis);
   pl->off_w = o;
   o = align_up(o + sizeof(float) * (size_t)pl->total_vis);
+  pl->score_bytes = o;
+  // The bf16 greedy's row skipping keeps up to kRootsPerRequest feature rows per
+  // request (min(k_b, kRootsPerRequest) rounded up to whole groups of 16, each row
+  // padded to whole 64-element blocks) and a table of bounds per root.
+  pl->root_rows = 0;
+  const bool sel_scratch = p->dtype == LAST_DTYPE_BF16 && p->feat_dim >= 8 &&
+                           p->feat_dim % 8 == 0 && p->feat_dim <= kMaxFeatDim;
+  auto root_cap = [&](int b) {
+    return (std::min(p->cu_keep[b + 1] - p->cu_keep[b], kRootsPerRequest) + 15) / 16 * 16;
+  };
+  if (sel_scratch)
+    for (int b = 0; b < B; ++b) pl->root_rows += root_cap(b);
+  pl->off_roots = o;
+  o = align_up(o + (size_t)pl->root_rows * (size_t)((std::max(p->feat_dim, 0) + 63) / 64) * 128);
+  pl->off_rtab = o;
+  o = align_up(o + (size_t)pl->root_rows * kRootTableCols * sizeof(float));
   pl->total_bytes = o;
 
   // ---- host staging: [err words][meta][items][order], one copy ----
@@ -135,8 +152,11 @@ last_status make_plan(const last_problem *p, bool need_scores, bool need_select,
   int32_t *items = pl->host_blob.data() + pl->off_items / 4;
   int32_t *order = pl->host_blob.data() + pl->off_order / 4;
   int chunk = 0;
+  long long root_off = 0;
   for (int b = 0; b < B; ++b) {
     int32_t *m = meta + b * kMetaFields;
+    m[kRootOff] = (int32_t)root_off;
+    if (sel_scratch) root_off += root_cap(b);
     m[kVisOff] = p->cu_vis[b];
     m[kNumVis] = p->cu_vis[b + 1] - p->cu_vis[b];
     m[kKeepOff] = p->cu_keep[b];
@@ -168,13 +188,13 @@ last_status make_plan(const last_problem *p, bool need_scores, bool need_select,
 
 namespace {
 
-last_status check_ws(const Plan &pl, const void *ws, size_t ws_bytes) {
+last_status check_ws(const Plan &pl, const void *ws, size_t ws_bytes, bool scores_only = false) {
   if (ws == nullptr) return fail(LAST_ERR_INVALID_ARG, "workspace is NULL");
   if ((reinterpret_cast<uintptr_t>(ws) & (kAlign - 1)) != 0)
     return fail(LAST_ERR_INVALID_ARG, "workspace must be 256-byte aligned");
-  if (ws_bytes < pl.total_bytes)
-    return fail(LAST_ERR_WORKSPACE_TOO_SMALL,
-                "workspace needs " + std::to_string(pl.total_bytes) + " bytes");
+  const size_t need = scores_only ? pl.score_bytes : pl.total_bytes;
+  if (ws_bytes < need)
+    return fail(LAST_ERR_WORKSPACE_TOO_SMALL, "workspace needs " + std::to_string(need) + " bytes");
   return LAST_OK;
 }
 
@@ -237,7 +257,7 @@ last_status last_scores(const last_problem *p, const void *q, const void *k, flo
   Plan pl;
   last_status st = make_plan(p, true, false, &pl);
   if (st != LAST_OK) return st;
-  if ((st = check_ws(pl, ws, ws_bytes)) != LAST_OK) return st;
+  if ((st = check_ws(pl, ws, ws_bytes, true)) != LAST_OK) return st;
   if (pl.total_vis > 0 && (q == nullptr || k == nullptr || w_out == nullptr))
     return fail(LAST_ERR_INVALID_ARG, "q, k and w_out are required");
   if (!aligned16(q) || !aligned16(k)) return fail(LAST_ERR_INVALID_ARG, "q and k must be 16-byte aligned");
@@ -305,8 +325,12 @@ last_status last_select_topk(const last_problem *p, const float *w, const void *
 last_status last_gather(const last_problem *p, const void *x, const int32_t *idx, void *x_out,
                         void *ws, size_t ws_bytes, void *stream) {
   Plan pl;
-  last_status st = make_plan(p, false, true, &pl);
+  // Eq. 12 is a row copy: only the row width must suit the kernel's 16-byte copies
+  // (the selection's own feature-width limit does not apply)
+  last_status st = make_plan(p, false, false, &pl);
   if (st != LAST_OK) return st;
+  if (p->feat_dim < 8 || p->feat_dim % 8 != 0)
+    return fail(LAST_ERR_INVALID_ARG, "feat_dim must be a positive multiple of 8");
   if ((st = check_ws(pl, ws, ws_bytes)) != LAST_OK) return st;
   if (pl.total_keep > 0 && (x == nullptr || idx == nullptr || x_out == nullptr))
     return fail(LAST_ERR_INVALID_ARG, "x, idx and x_out are required");

@@ -21,6 +21,7 @@ enum MetaField : int {
   kKeepOff,        // cu_keep[b]
   kNumKeep,        // k_b
   kChunkBase,      // first score chunk of request b
+  kRootOff,        // first row of request b in the selection's root rows
   kMetaFields
 };
 
@@ -28,6 +29,8 @@ constexpr int kScoreThreads = 256;
 constexpr int kTokenTile = kScoreThreads;   // visual tokens per score_tokens_kernel CTA
 constexpr int kMaxGroup = 8;         // q-heads per kv-head supported by the scoring kernel
 constexpr int kMaxFeatDim = 2048;    // selection keeps x_j in 64 fp32 registers per lane
+constexpr int kRootsPerRequest = 1024;   // root rows per request (the selection's kMaxRoots)
+constexpr int kRootTableCols = 32;       // bound-table columns per root (the selection's kMaxAccept)
 constexpr int kSelectWarps = 8;
 constexpr int kGatherThreads = 256;
 
@@ -48,6 +51,10 @@ struct Plan {
   // workspace byte offsets
   size_t off_err = 0, off_meta = 0, off_items = 0, off_order = 0;
   size_t off_stats = 0, off_zlog = 0, off_w = 0, total_bytes = 0;
+  // bf16 selection scratch: root rows [root_rows][dv] and the bound table
+  // [root_rows][kRootTableCols] (after the scoring scratch; score_bytes excludes them)
+  size_t off_roots = 0, off_rtab = 0, score_bytes = 0;
+  long long root_rows = 0;
   // host staging (error word, meta rows, score items, selection order) in ws order
   std::vector<int32_t> host_blob;
   size_t blob_bytes = 0;  // bytes from off_meta to the end of the order array
@@ -61,6 +68,7 @@ last_status make_plan(const last_problem *p, bool need_scores, bool need_select,
                       const int32_t *seq_len = nullptr);
 
 void set_error(const std::string &msg);
+std::string get_error();   // the message last_error_message() returns on this thread
 
 // Kernel launchers (return cudaSuccess or the launch error).
 cudaError_t launch_scores(const Plan &pl, const void *q, const void *k, float *w_out,

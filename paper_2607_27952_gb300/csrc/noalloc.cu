@@ -70,8 +70,8 @@ extern "C" last_status last_scores_noalloc(const last_problem *p, const void *q,
   Plan pl;
   last_status st = make_plan(p, true, false, &pl);
   if (st != LAST_OK) return st;
-  if (pl.total_bytes > kNoAllocScratchBytes) {
-    set_error("last_scores_noalloc: this problem needs " + std::to_string(pl.total_bytes) +
+  if (pl.score_bytes > kNoAllocScratchBytes) {
+    set_error("last_scores_noalloc: this problem needs " + std::to_string(pl.score_bytes) +
               " bytes of scratch, more than the library's fixed " +
               std::to_string(kNoAllocScratchBytes) + " bytes; use last_scores with a workspace");
     return LAST_ERR_UNSUPPORTED;

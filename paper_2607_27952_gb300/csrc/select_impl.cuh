@@ -63,6 +63,44 @@ constexpr int kTcBoxBytes = kTcBM * kTcBK * 2;     // one A box (128 rows x 64 e
 constexpr int kTmemCols = 512;                     // TMEM columns per SM
 constexpr int kGramChains = 4;                     // accumulators of the list's Gram
 
+// Row skipping by the triangle inequality (tensor-core variant).  Every accepted
+// centre is either a "root" (no earlier root within chordal distance kTriTau) or is
+// attached to its nearest root R with an upper bound e >= rho(centre, R), where
+// rho(a, b) = |a/|a| - b/|b|| = sqrt(2 (1 - cos(a, b))) is the chordal metric on the
+// unit sphere.  Token i with nearest centre o (delta_i = d(i, o)) and o's root R
+// satisfies, for a new centre c,
+//   rho(i, c) >= rho(R, c) - rho(R, o) - rho(o, i) >= rho_lb(R, c) - e_o - rho_up(i),
+// so rho_lb(R, c) >= 2 rho_up(i) + e_o proves d(i, c) >= delta_i and c cannot lower
+// delta_i.  The bounds carry the rounding of every computed distance (kTriEpsC for
+// the canonical fp32 order against exact arithmetic, plus the tensor-core bound for
+// the root table) and are evaluated with directed rounding, so a skipped pair is
+// one whose canonical fminf would have left delta_i unchanged: the selection stays
+// bit-identical.  Rows outside a safe norm range (no underflow or overflow in the
+// canonical dot) are never skipped.
+constexpr int kMaxRoots = kRootsPerRequest;        // roots per request (workspace rows)
+// Candidate list of the tensor-core variant: each CTA keeps up to kDeep of its
+// highest keys w~_i delta_i (sorted) and a bound theta that every other token's key
+// stays below (keys never increase).  After a round the entries still above theta
+// are exactly the CTA's top keys, so the CTA re-ranks all of its tokens only when
+// fewer than the published count remain.
+constexpr int kDeep = 64;
+static_assert(kMaxAccept == kRootTableCols, "the bound table has one column per accepted centre");
+constexpr int kRootGroup = 16;                     // roots per group: the table MMA's N
+// Root rows are stored in groups of 16 in the MMA's shared-memory image: K block kb
+// of the group at kb * 2048, row i at i * 128, 16-byte chunk c at (c ^ (i % 8)) * 16
+// (K-major, 128-byte swizzle).  One bulk copy then moves any run of K blocks.
+constexpr int kRootGroupKbBytes = kRootGroup * 128;
+// The root table streams through the update's ring, cut into kTabSt stages with
+// barriers of their own (the update's stages are idle while it runs), so that
+// many small bulk copies are in flight while the candidate list is processed.
+constexpr int kTabSt = 8;
+constexpr float kTriTau = 0.5f;                    // chordal radius that makes a centre a root
+// |canonical fp32 distance - exact distance| for rows of norm in [2^-50, 2^50] and
+// d_v <= 2048: the dot's at most 64 fmas per lane and 5 butterfly additions give
+// 69 u relative to |x_i||x_j|, each reciprocal norm 36.5 u, the two scalings and the
+// subtraction 3 u more: 8.9e-6 in all (u = 2^-24); taken with a 3x margin.
+constexpr float kTriEpsC = 3e-5f;
+
 struct SelectArgs {
   CUtensorMap tmap;      // X as [total_vis][dv] bf16, box 64 x 128, 128-byte swizzle (tc only)
   const void *x;
@@ -81,13 +119,19 @@ struct SelectArgs {
   int tc_stages;         // tc: TMA ring depth (2..kTcMaxStages)
   int tc_kps;            // tc: K blocks (boxes) per ring stage
   float tc_eps;          // tc: bound on |tensor-core distance - canonical distance|
+  // triangle-inequality skipping (tc only)
+  char *roots;           // root row groups: request b's from row meta kRootOff (a multiple of 16)
+  float *rtab;           // per round: rho lower bounds [root row][kMaxAccept]
+  int tri;               // 1: skip rows by the triangle inequality
+  int root_cap;          // roots per request (<= kMaxRoots, <= s_cap * csize)
+  float tri_eps_x;       // bound on |root-table distance - exact distance| (tc_eps + kTriEpsC)
 };
 
 // Shared-memory carve-up, identical on host (sizing) and device.
 struct SelectSmem {
   size_t aring, xcache, cbuf, ring, blk, w, r, dl, list, sel, wtop, pub_key, pub_f, lp_key,
       lp_f, lp_idx, lp_row, pair, acc, misc, bar, cnt, tbar, tslot, fidx, fmask, fcnt, gram, plist,
-      total;
+      oroot, oe, mr, rootr, part, croot, ce, rowj, nrl, deep, total;
 };
 // K blocks of kTcBK elements covering a feature row.
 __host__ __device__ inline int tc_kblocks(int dv) { return (dv + kTcBK - 1) / kTcBK; }
@@ -102,7 +146,8 @@ __host__ __device__ inline int blocks_per_warp(int tpc_max, int tb) {
 }
 __host__ __device__ inline SelectSmem select_smem(int cache_rows, int row_bytes, int tpc_max,
                                                   int ring, int tb, int elem, int lcap,
-                                                  int tc = 0, int stages = 0, int kps = 1) {
+                                                  int tc = 0, int stages = 0, int kps = 1,
+                                                  int roots = 0) {
   SelectSmem s;
   size_t o = 0;
   if (tc) {
@@ -139,13 +184,28 @@ __host__ __device__ inline SelectSmem select_smem(int cache_rows, int row_bytes,
   s.bar = o; o += sizeof(unsigned long long);
   s.cnt = o; o += sizeof(int) * kMaxCluster;
   o = align16(o);
-  s.tbar = o; o += tc ? sizeof(unsigned long long) * (2 * kTcMaxStages + 2) : 0;
+  s.tbar = o; o += tc ? sizeof(unsigned long long) * (2 * kTcMaxStages + 4 + 2 * kTabSt) : 0;
   s.tslot = o; o += tc ? 16 : 0;
   s.fidx = o; o += tc ? align16(sizeof(int) * tpc_max) : 0;
   s.fmask = o; o += tc ? align16(sizeof(uint32_t) * tpc_max) : 0;
   s.fcnt = o; o += tc ? 16 : 0;
   s.gram = o; o += tc ? sizeof(float) * kLcap * kLcap : 0;       // list Gram (tensor cores)
   s.plist = o; o += tc ? align16(sizeof(int) * (kMaxPairs + 1)) : 0;   // pairs to evaluate
+  // triangle-inequality state: per token the root of its nearest centre and the bound
+  // e of that centre; per root the round's smallest rho lower bound and its 1/|x|;
+  // per accepted centre its root and e; the cluster's partial nearest-root searches
+  // (sized 0 when the launch does not skip rows: roots == 0)
+  const bool tri = tc && roots > 0;
+  s.oroot = o; o += tri ? align16(sizeof(int) * tpc_max) : 0;
+  s.oe = o; o += tri ? align16(sizeof(float) * tpc_max) : 0;
+  s.mr = o; o += tri ? align16(sizeof(float) * roots) : 0;
+  s.rootr = o; o += tri ? align16(sizeof(float) * roots) : 0;
+  s.part = o; o += tri ? sizeof(float2) * kMaxCluster * kMaxAccept : 0;
+  s.croot = o; o += tri ? sizeof(int) * kMaxAccept : 0;
+  s.ce = o; o += tri ? sizeof(float) * kMaxAccept : 0;
+  s.rowj = o; o += tri ? sizeof(int) * kLcap : 0;
+  s.nrl = o; o += tri ? sizeof(int2) * (kMaxAccept + 1) : 0;
+  s.deep = o; o += tc ? sizeof(unsigned long long) * kDeep + 16 : 0;   // candidate list + flag
   s.total = align16(o) + 1024;   // slack for aligning the base to 1024 bytes
   return s;
 }
@@ -204,6 +264,13 @@ __device__ __forceinline__ void warp_argmax(unsigned long long &key, int &payloa
   }
 }
 
+// maximum over the warp of a 64-bit key (every lane returns it)
+__device__ __forceinline__ unsigned long long warp_max_u64(unsigned long long v) {
+  const uint32_t hi = __reduce_max_sync(0xffffffffu, (uint32_t)(v >> 32));
+  const uint32_t lo = __reduce_max_sync(0xffffffffu, (uint32_t)(v >> 32) == hi ? (uint32_t)v : 0u);
+  return ((unsigned long long)hi << 32) | lo;
+}
+
 // descending top-W list held in (warp-uniform) registers
 template <int W>
 struct TopList {
@@ -223,6 +290,33 @@ struct TopList {
   }
 };
 
+// ---- triangle-inequality bounds (directed rounding: each is a true bound) ----
+// 1/|x| of a row whose canonical dot products obey the kTriEpsC bound
+__device__ __forceinline__ bool tri_in_range(float r) { return r >= 0x1p-50f && r <= 0x1p50f; }
+// upper bound on rho(i, o) from delta_i = d(i, o) (canonical), +inf when unbounded
+__device__ __forceinline__ float tri_rho_up(float delta) {
+  if (!(delta <= 4.0f)) return INFINITY;
+  return __fsqrt_ru(__fmul_ru(2.0f, fmaxf(__fadd_ru(delta, kTriEpsC), 0.0f)));
+}
+// lower bound on rho(a, b) from a computed distance d with |d - exact| <= eps
+__device__ __forceinline__ float tri_rho_lb(float d, float eps) {
+  const float v = __fsub_rd(d, eps);
+  return v > 0.0f ? __fsqrt_rd(__fmul_rd(2.0f, v)) : 0.0f;   // NaN -> 0 (never skips)
+}
+// upper bound on rho(a, b) from a computed distance d with |d - exact| <= eps
+__device__ __forceinline__ float tri_rho_ub(float d, float eps) {
+  const float v = __fadd_ru(d, eps);
+  if (!(v <= 4.0f)) return INFINITY;
+  return __fsqrt_ru(__fmul_ru(2.0f, fmaxf(v, 0.0f)));
+}
+// rho_lb(R, c) >= 2 rho_up(i) + e_o: c cannot lower delta_i
+__device__ __forceinline__ float tri_need(float delta, float e) {
+  return __fadd_ru(__fmul_ru(2.0f, tri_rho_up(delta)), e);
+}
+__device__ __forceinline__ void fence_proxy_async_global() {
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+
 template <typename T, int NCH, int TB, bool TC>
 __global__ void __launch_bounds__(kSelThreads, 1)
 select_kernel(const __grid_constant__ SelectArgs a) {
@@ -237,9 +331,11 @@ select_kernel(const __grid_constant__ SelectArgs a) {
   const int32_t *m = a.meta + b * kMetaFields;
   const int voff = m[kVisOff], N = m[kNumVis], koff = m[kKeepOff], K = m[kNumKeep];
   if (K == 0) return;  // the whole cluster leaves together; no DSMEM traffic yet
+  const int rootoff = m[kRootOff];
 
   const SelectSmem S = select_smem(a.cache_rows, a.row_bytes, a.tpc_max, a.ring, TB, (int)sizeof(T),
-                                   a.lcap, TC ? 1 : 0, TC ? a.tc_stages : 0, TC ? a.tc_kps : 1);
+                                   a.lcap, TC ? 1 : 0, TC ? a.tc_stages : 0, TC ? a.tc_kps : 1,
+                                   TC && a.tri ? a.root_cap : 0);
   {
     // The host sizes the launch with the same plan; should they ever disagree, every
     // CTA of every cluster leaves here together (before any cluster barrier)
@@ -273,6 +369,19 @@ select_kernel(const __grid_constant__ SelectArgs a) {
   int *acc_s = reinterpret_cast<int *>(smem + S.acc);
   unsigned long long *misc = reinterpret_cast<unsigned long long *>(smem + S.misc);
   int *cnt_s = reinterpret_cast<int *>(smem + S.cnt);
+  // triangle-inequality state (tensor-core variant)
+  const bool tri = TC && a.tri != 0;
+  int *oroot_s = reinterpret_cast<int *>(smem + S.oroot);
+  float *oe_s = reinterpret_cast<float *>(smem + S.oe);
+  float *mr_s = reinterpret_cast<float *>(smem + S.mr);
+  float *rootr_s = reinterpret_cast<float *>(smem + S.rootr);
+  float2 *part_s = reinterpret_cast<float2 *>(smem + S.part);   // [kMaxCluster][kMaxAccept]
+  int *croot_s = reinterpret_cast<int *>(smem + S.croot);
+  float *ce_s = reinterpret_cast<float *>(smem + S.ce);
+  int *rowj_s = reinterpret_cast<int *>(smem + S.rowj);
+  int2 *nrl_s = reinterpret_cast<int2 *>(smem + S.nrl);         // new roots: (root id, token)
+  const int rcap = tri ? min(a.root_cap, K) : 0;
+  int nroot = 0;   // roots of this request (the same in every CTA of the cluster)
 
   const int tpr = (N + C - 1) / C;  // tokens per CTA for this request
   const int lo = min(N, (int)rank * tpr), hi = min(N, lo + tpr);
@@ -292,6 +401,11 @@ select_kernel(const __grid_constant__ SelectArgs a) {
   unsigned long long *tempty = tfull + kTcMaxStages;
   unsigned long long *tdone = tempty + kTcMaxStages;
   unsigned long long *tpair = tdone + 1;
+  unsigned long long *ttab = tpair + 1;   // the round's root table is in TMEM
+  unsigned long long *txb = ttab + 1;     // rows of the exact step (bulk copies)
+  unsigned long long *tbf = txb + 1;      // root-table stages: landed
+  unsigned long long *tbe = tbf + kTabSt; // root-table stages: consumed by the MMAs
+  uint32_t txph = 0;
   if (threadIdx.x == 0) {
     mbar_init(bar, 1);
     if constexpr (TC) {
@@ -301,6 +415,12 @@ select_kernel(const __grid_constant__ SelectArgs a) {
       }
       mbar_init(tdone, 1);
       mbar_init(tpair, 1);
+      mbar_init(ttab, 1);
+      mbar_init(txb, 1);
+      for (int i = 0; i < kTabSt; ++i) {
+        mbar_init(&tbf[i], 1);
+        mbar_init(&tbe[i], 1);
+      }
     }
     fence_mbar_init();
   }
@@ -313,6 +433,10 @@ select_kernel(const __grid_constant__ SelectArgs a) {
     w_s[t] = a.w[voff + lo + t];
     dl_s[t] = INFINITY;
     sel_s[t] = (K == N) ? 1 : 0;
+    if (tri) {
+      oroot_s[t] = -1;      // no nearest centre yet: never skipped
+      oe_s[t] = INFINITY;
+    }
   }
   if (ncache > 0) {
     mbar_wait_bounded(bar, phase, a.err, kErrTimeout);
@@ -355,8 +479,103 @@ select_kernel(const __grid_constant__ SelectArgs a) {
     // Merge the warps' lists into the CTA's kTop best and publish them (key and
     // {delta, w, r}) to every CTA of the cluster, into buffer `par`.
     unsigned long long *top5 = misc + 4;  // misc[4..4+kTop)
+    unsigned long long *dkey = reinterpret_cast<unsigned long long *>(smem + S.deep);
+    int *drescan = reinterpret_cast<int *>(smem + S.deep + sizeof(unsigned long long) * kDeep);
+    unsigned long long d_theta = 0ull;   // warp 0: bound on every key outside dkey
+    int d_n = 0;                         // warp 0: entries of dkey
+    // warp 0: the list holds keys w~ delta (not the seed round's w~ alone: a key w~
+    // delta can exceed w~ when delta > 1, so that first list bounds nothing later)
+    bool d_bounds = false;
+    // warp 0: the union of the warps' ranked lists -> the candidate list.  Every
+    // token a warp left out has a key below that warp's last entry, so the union's
+    // entries above the largest such entry are the CTA's top keys, in order.
+    auto deep_rebuild = [&](bool bounds) {
+      if (warp != 0) return;
+      d_bounds = bounds;
+      constexpr int nk = kSelectWarps * kTop;
+      constexpr int kPerLane = (nk + 31) / 32;
+      unsigned long long kl[kPerLane];
+      int rl[kPerLane];
+#pragma unroll
+      for (int j = 0; j < kPerLane; ++j) {
+        kl[j] = lane + 32 * j < nk ? wtop[lane + 32 * j] : 0ull;
+        rl[j] = 0;
+      }
+      unsigned long long th = lane < kSelectWarps ? wtop[lane * kTop + kTop - 1] : 0ull;
+      {
+        const uint32_t hi = __reduce_max_sync(0xffffffffu, (uint32_t)(th >> 32));
+        const uint32_t lo_ = __reduce_max_sync(0xffffffffu, (uint32_t)(th >> 32) == hi ? (uint32_t)th : 0u);
+        th = ((unsigned long long)hi << 32) | lo_;
+      }
+#pragma unroll
+      for (int f = 0; f < nk; ++f) {
+        const unsigned long long kf = wtop[f];
+#pragma unroll
+        for (int j = 0; j < kPerLane; ++j) rl[j] += kf > kl[j] ? 1 : 0;
+      }
+      int above = 0;
+      unsigned long long cut = 0ull;
+#pragma unroll
+      for (int j = 0; j < kPerLane; ++j) {
+        const bool up = kl[j] > th;
+        above += __popc(__ballot_sync(0xffffffffu, up));
+        if (up && rl[j] < kDeep) dkey[rl[j]] = kl[j];
+        if (up && rl[j] == kDeep) cut = kl[j];
+      }
+      {
+        const uint32_t hi = __reduce_max_sync(0xffffffffu, (uint32_t)(cut >> 32));
+        const uint32_t lo_ = __reduce_max_sync(0xffffffffu, (uint32_t)(cut >> 32) == hi ? (uint32_t)cut : 0u);
+        cut = ((unsigned long long)hi << 32) | lo_;
+      }
+      d_n = min(above, kDeep);
+      d_theta = above > kDeep ? cut : th;
+      __syncwarp();
+    };
+    // warp 0, after an update: the list's keys from the new deltas; entries that fell
+    // to theta or below (or were selected) leave it.  Sets *drescan when fewer than
+    // the published count remain while other tokens exist.
+    auto deep_refresh = [&]() {
+      if (warp != 0) return;
+      if (!d_bounds) {
+        if (lane == 0) *drescan = 1;
+        __syncwarp();
+        return;
+      }
+      unsigned long long k[2];
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const int e = lane + 32 * h;
+        k[h] = 0ull;
+        if (e < d_n) {
+          const int gi = key_index(dkey[e]);
+          const int t = gi - lo;
+          const unsigned long long nk = sel_s[t] ? 0ull : argmax_key(__fmul_rn(w_s[t], dl_s[t]), gi);
+          k[h] = nk > d_theta ? nk : 0ull;
+        }
+      }
+      int r0 = 0, r1 = 0;
+#pragma unroll 8
+      for (int src = 0; src < 32; ++src) {
+        const unsigned long long a0 = shfl_u64(k[0], src), a1 = shfl_u64(k[1], src);
+        r0 += (a0 > k[0] ? 1 : 0) + (a1 > k[0] ? 1 : 0);
+        r1 += (a0 > k[1] ? 1 : 0) + (a1 > k[1] ? 1 : 0);
+      }
+      const int kept = __popc(__ballot_sync(0xffffffffu, k[0] != 0ull)) +
+                       __popc(__ballot_sync(0xffffffffu, k[1] != 0ull));
+      __syncwarp();
+      if (k[0] != 0ull) dkey[r0] = k[0];
+      if (k[1] != 0ull) dkey[r1] = k[1];
+      d_n = kept;
+      if (lane == 0) *drescan = (d_n >= a.mc + 1 || d_theta == 0ull) ? 0 : 1;
+      __syncwarp();
+    };
     auto publish = [&](int par) {
       if (warp == 0) {
+        if constexpr (TC) {
+          // the candidate list holds the CTA's top keys (at least mc + 1 of them, or
+          // every live token)
+          if (lane < kTop) top5[lane] = lane < d_n ? dkey[lane] : 0ull;
+        } else {
         constexpr int nk = kSelectWarps * kTop;   // the warps' ranked keys
         constexpr int kPerLane = (nk + 31) / 32;
         static_assert(kPerLane <= 5, "publish ranks at most 160 keys");
@@ -378,6 +597,7 @@ select_kernel(const __grid_constant__ SelectArgs a) {
 #pragma unroll
         for (int j = 0; j < kPerLane; ++j)
           if (kl[j] != 0ull && rl[j] < kTop) top5[rl[j]] = kl[j];
+        }
         __syncwarp();
         if (lane < C) {
           for (int i = 0; i <= a.mc; ++i) {
@@ -631,7 +851,7 @@ select_kernel(const __grid_constant__ SelectArgs a) {
       *abort_w = 1u;
       return false;
     };
-    auto update_tc = [&](int nA) {
+    auto update_tc = [&](int nA, bool tri_round) {
       const int nkb = tc_kblocks(dv);
       char *aring = reinterpret_cast<char *>(smem + S.aring);
       int *fidx = reinterpret_cast<int *>(smem + S.fidx);
@@ -644,6 +864,87 @@ select_kernel(const __grid_constant__ SelectArgs a) {
       tc_fence_before();
       __syncthreads();
       tc_fence_after();
+      // 1b. triangle test: a token survives unless the round's root table proves that
+      //     no accepted centre can lower its delta.  A survivor is "hard" when no
+      //     bound can exclude any centre for it (2 rho_up + e above 2, the largest
+      //     chordal distance: its delta is still near 1); its pairs all need a
+      //     distance.  With few survivors their pairs are evaluated exactly (step 4)
+      //     without streaming X; otherwise the dense tensor-core pass decides every
+      //     pair.  The choice compares the bytes the dense pass streams with the
+      //     survivors' rows plus their exact pairs (about 5/16 of a row each).
+      bool dense = true;
+      if (tri_round) {
+        if (threadIdx.x == 0) fcnt[1] = 0;
+        __syncthreads();
+        for (int t0 = warp * 32; t0 < nloc; t0 += kSelThreads) {
+          const int t = t0 + lane;
+          bool act = false, hard = false;
+          if (t < nloc && !sel_s[t]) {
+            act = hard = true;
+            const int R = oroot_s[t];
+            if (R >= 0 && tri_in_range(r_s[t])) {
+              const float nd = tri_need(dl_s[t], oe_s[t]);
+              act = !(mr_s[R] >= nd);
+              hard = !(nd <= 2.0f);
+            }
+          }
+          const unsigned bal = __ballot_sync(0xffffffffu, act);
+          const unsigned hb = __ballot_sync(0xffffffffu, act && hard);
+          int base = 0;
+          if (lane == 0 && bal != 0u) {
+            base = atomicAdd(fcnt, __popc(bal));
+            if (hb != 0u) atomicAdd(fcnt + 1, __popc(hb));
+          }
+          base = __shfl_sync(0xffffffffu, base, 0);
+          if (act) fidx[base + __popc(bal & ((1u << lane) - 1u))] = t;
+        }
+        __syncthreads();
+        const int nact = fcnt[0], nhard = fcnt[1];
+        const long long pair_bytes = (long long)dv * 5 / 16;
+        const long long sparse_cost = (long long)nact * rb * 5 / 4 +
+                                      ((long long)nhard * nA + 2LL * (nact - nhard)) * pair_bytes;
+        dense = sparse_cost > (long long)nloc * rb;
+        __syncthreads();   // every thread has read the counts
+        if (dense) {
+          if (threadIdx.x == 0) *fcnt = 0;
+        } else {
+          // the centres the survivor's root bound does not exclude (table rows written
+          // by the slice owners before the last cluster barrier; read past L1); four
+          // survivors per warp at a time keep their table loads in flight together
+          for (int f0 = warp; f0 < nact; f0 += 4 * kSelectWarps) {
+            float tv[4], nd[4];
+            bool chk[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+              const int f = f0 + u * kSelectWarps;
+              chk[u] = false;
+              tv[u] = 0.f;
+              nd[u] = 0.f;
+              if (f < nact && lane < nA) {
+                const int t = fidx[f];
+                const int R = oroot_s[t];
+                if (R >= 0 && tri_in_range(r_s[t])) {
+                  nd[u] = tri_need(dl_s[t], oe_s[t]);
+                  if (nd[u] <= 2.0f) {
+                    chk[u] = true;
+                    tv[u] = __ldcg(a.rtab + (size_t)(rootoff + R) * kMaxAccept + lane);
+                  }
+                }
+              }
+            }
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+              const int f = f0 + u * kSelectWarps;
+              if (f < nact) {
+                const unsigned msk = __ballot_sync(0xffffffffu, lane < nA && !(chk[u] && tv[u] >= nd[u]));
+                if (lane == 0) fmask[f] = msk;
+              }
+            }
+          }
+        }
+        __syncthreads();
+      }
+      if (dense) {
       // 2. TMA producer (thread 0) and MMA issuer (thread 32)
       const int ntile = (nloc + kTcBM - 1) / kTcBM;
       // a ring stage holds kps consecutive K blocks of one tile (one barrier, one
@@ -722,12 +1023,16 @@ select_kernel(const __grid_constant__ SelectArgs a) {
       }
       tc_fence_before();
       __syncthreads();
-      // 4. exact canonical distances for the flagged pairs (a warp per token, two
-      //    tokens' rows in flight)
+      }   // dense
+      // 4. exact canonical distances for the flagged pairs.  The flagged tokens' rows
+      //    are bulk-copied into the ring (idle now) in batches, every copy of a batch
+      //    in flight at once; then a warp per token evaluates its pairs from shared
+      //    memory in the canonical order.
       const int nf = *fcnt;
       auto exact_token = [&](int t, unsigned msk, const U4 *xv) {
         const float ri = r_s[t];
         float dl = dl_s[t];
+        int own = -1;   // the accepted centre that last lowered delta (nearest centre)
         while (msk) {
           const int j = __ffs(msk) - 1;
           msk &= msk - 1;
@@ -748,25 +1053,46 @@ select_kernel(const __grid_constant__ SelectArgs a) {
             }
           }
           const float dot = butterfly_sum(acc);
-          dl = fminf(dl, __fsub_rn(1.0f, __fmul_rn(__fmul_rn(dot, ri), lp_f[acc_s[j] * 3 + 2])));
+          const float d = __fsub_rn(1.0f, __fmul_rn(__fmul_rn(dot, ri), lp_f[acc_s[j] * 3 + 2]));
+          if (d < dl) own = j;
+          dl = fminf(dl, d);
         }
-        if (lane == 0) dl_s[t] = dl;
+        if (lane == 0) {
+          dl_s[t] = dl;
+          if (tri && own >= 0) {
+            oroot_s[t] = croot_s[own];
+            oe_s[t] = ce_s[own];
+          }
+        }
       };
-      for (int f = warp; f < nf; f += 2 * kSelectWarps) {
-        const int f2 = f + kSelectWarps;
-        const int t0 = fidx[f], t1 = f2 < nf ? fidx[f2] : t0;
-        U4 xa[NCH], xb[NCH];
-#pragma unroll
-        for (int g = 0; g < NCH; ++g) {
-          const int col = 256 * g + 8 * lane;
-          xa[g] = col < dv ? ldg(xg + (long long)t0 * rb + col * 2) : U4{0, 0, 0, 0};
-          xb[g] = col < dv ? ldg(xg + (long long)t1 * rb + col * 2) : U4{0, 0, 0, 0};
+      const int per_batch = min(nstage * a.tc_kps * kTcBoxBytes / rb, 64);
+      for (int b0 = 0; b0 < nf; b0 += per_batch) {
+        const int nb = min(per_batch, nf - b0);
+        if (threadIdx.x == 0) {
+          fence_proxy_async_smem();   // the last batch's reads precede these writes
+          mbar_expect_tx(txb, (uint32_t)(nb * rb));
+          for (int i = 0; i < nb; ++i)
+            bulk_g2s(aring + (long long)i * rb, xg + (long long)fidx[b0 + i] * rb, (uint32_t)rb, txb);
         }
-        exact_token(t0, fmask[f], xa);
-        if (f2 < nf) exact_token(t1, fmask[f2], xb);
+        mbar_wait_bounded(txb, txph, a.err, kErrTimeout);
+        txph ^= 1u;
+        for (int f = b0 + warp; f < b0 + nb; f += kSelectWarps) {
+          const uint32_t row = smem_addr(aring + (long long)(f - b0) * rb);
+          U4 xv[NCH];
+#pragma unroll
+          for (int g = 0; g < NCH; ++g) {
+            const int col = 256 * g + 8 * lane;
+            xv[g] = col < dv ? lds32(row + (uint32_t)(col * 2)) : U4{0, 0, 0, 0};
+          }
+          exact_token(fidx[f], fmask[f], xv);
+        }
+        __syncthreads();
       }
+      // 5. the candidate list from the new deltas; all tokens are re-ranked only when
+      //    too few of its entries are still known to lead
+      deep_refresh();
       __syncthreads();
-      // 5. keys of the unselected tokens -> the warp's ranked list for the next round
+      if (*drescan == 0) return;
       TopList<kTop> tl;
       tl.clear();
       for (int t0 = warp * 32; t0 < nloc; t0 += kSelectWarps * 32) {
@@ -788,11 +1114,14 @@ select_kernel(const __grid_constant__ SelectArgs a) {
 #pragma unroll
         for (int i = 0; i < kTop; ++i) wtop[warp * kTop + i] = tl.k[i];
       }
+      __syncthreads();
+      deep_rebuild(true);
     };
-    auto update = [&](int nA) {
+    auto update = [&](int nA, bool tri_round) {
       if constexpr (TC) {
-        update_tc(nA);
+        update_tc(nA, tri_round);
       } else {
+        (void)tri_round;
         if (nA <= 4) update_nb(std::integral_constant<int, 4>{}, nA);
         else if (nA <= 8) update_nb(std::integral_constant<int, 8>{}, nA);
         else if (nA <= 12) update_nb(std::integral_constant<int, 12>{}, nA);
@@ -800,7 +1129,197 @@ select_kernel(const __grid_constant__ SelectArgs a) {
       }
     };
 
+    // ---- triangle-inequality bookkeeping (tensor-core variant) ----
+    // Each round the cluster's CTAs split the request's roots: CTA `rank` takes roots
+    // [tr_s0, tr_s0 + tr_cnt) and forms their dot products with every list row on the
+    // tensor cores (A = the list rows in cbuf, B = the roots' rows streamed through
+    // the ring by bulk copies, tr_kbps K blocks of one group per ring stage; fp32
+    // accumulators in TMEM columns [0, tr_w), which the update's tiles reuse later).
+    int tr_s0 = 0, tr_cnt = 0, tr_w = 0, tr_kbps = 1, tr_nts = 0, tr_pre = 0;
+    int tr_issued = 0, tr_mma = 0;   // thread 64: stages issued; thread 32: stages consumed
+    uint32_t tb_pit = 0, tb_mit = 0;  // their running stage counters (barrier phases)
+    uint32_t tc_tph = 0;   // root-table phase
+    const int tab_sb = (nstage * a.tc_kps * kTcBoxBytes / kTabSt) / kRootGroupKbBytes * kRootGroupKbBytes;
+    auto tri_slice = [&]() {
+      const int per = ((nroot + C - 1) / C + kRootGroup - 1) / kRootGroup * kRootGroup;
+      tr_s0 = min(nroot, (int)rank * per);
+      tr_cnt = min(nroot, tr_s0 + per) - tr_s0;
+      tr_w = per;
+      tr_kbps = tab_sb / kRootGroupKbBytes;   // K blocks of one group per stage
+      const int ngrp = (tr_cnt + kRootGroup - 1) / kRootGroup;
+      tr_nts = ngrp * ((tc_kblocks(dv) + tr_kbps - 1) / tr_kbps);
+      tr_pre = min(tr_nts, kTabSt);
+      tr_issued = 0;
+      tr_mma = 0;
+    };
+    // thread 64: bulk copies of table stages [tr_issued, upto) into the ring; stage s
+    // holds K blocks [kb0, kb0 + tr_kbps) of root group s / (stages per group).  A
+    // stage slot is reused once the MMAs of its previous stage are done; `block`
+    // false issues only what is free now.
+    auto table_load = [&](int upto, bool block) {
+      char *aring = reinterpret_cast<char *>(smem + S.aring);
+      const int nkb = tc_kblocks(dv);
+      const int spg = (nkb + tr_kbps - 1) / tr_kbps;
+      for (; tr_issued < upto; ++tr_issued, ++tb_pit) {
+        const int st = tb_pit % kTabSt;
+        if (tb_pit >= (uint32_t)kTabSt) {
+          const uint32_t par = ((tb_pit / kTabSt) - 1) & 1;
+          if (!block && !mbar_try_wait(&tbe[st], par)) break;
+          if (block && !twait(&tbe[st], par)) continue;
+        }
+        const int g = tr_issued / spg, kb0 = (tr_issued % spg) * tr_kbps, nb = min(tr_kbps, nkb - kb0);
+        const char *src = a.roots + (long long)(rootoff + tr_s0 + g * kRootGroup) * (nkb * 128) +
+                          (long long)kb0 * kRootGroupKbBytes;
+        mbar_expect_tx(&tbf[st], (uint32_t)(nb * kRootGroupKbBytes));
+        bulk_g2s(aring + st * tab_sb, src, (uint32_t)(nb * kRootGroupKbBytes), &tbf[st]);
+      }
+    };
+    // thread 32: the table's MMAs (N = 16 roots of one group into TMEM columns
+    // [16 g, 16 g + 16)) for stages that have landed; `block` waits for all of them
+    // and then commits to ttab
+    auto table_mma = [&](bool block) {
+      const int nkb = tc_kblocks(dv);
+      const int spg = (nkb + tr_kbps - 1) / tr_kbps;
+      const uint32_t aring_sa = smem_addr(smem + S.aring);
+      const uint32_t idesc = umma_idesc_bf16(kTcBM, kRootGroup);
+      for (; tr_mma < tr_nts; ++tr_mma, ++tb_mit) {
+        const int st = tb_mit % kTabSt;
+        const uint32_t par = (tb_mit / kTabSt) & 1;
+        if (!block && !mbar_try_wait(&tbf[st], par)) return;
+        const bool ok = !block || twait(&tbf[st], par);
+        tc_fence_after();
+        if (ok) {
+          const int g = tr_mma / spg, kb0 = (tr_mma % spg) * tr_kbps, nb = min(tr_kbps, nkb - kb0);
+          for (int q = 0; q < nb; ++q)
+#pragma unroll
+            for (int k = 0; k < kTcBK / 16; ++k)
+              umma_bf16(tmem + (uint32_t)(g * kRootGroup),
+                        umma_desc_sw128(cbuf_sa + (kb0 + q) * lcap * 128 + k * 32),
+                        umma_desc_sw128(aring_sa + st * tab_sb + q * kRootGroupKbBytes + k * 32),
+                        idesc, ((kb0 + q) | k) != 0 ? 1u : 0u);
+        }
+        umma_commit(&tbe[st]);
+      }
+      if (block) umma_commit(ttab);
+    };
+    // the table's service threads at a point where they are otherwise idle
+    auto table_poll = [&]() {
+      if (!tri || tr_nts == 0) return;
+      if (threadIdx.x == 32) table_mma(false);
+      else if (threadIdx.x == 64) table_load(tr_nts, false);
+    };
+    // warp 0 (TMEM lanes = cbuf rows): for every root of the slice, the lower bound
+    // rho_lb(R, c_j) per accepted centre into the global table, their minimum over
+    // the centres into every CTA's mr_s[R], and per centre the nearest root of the
+    // slice into every CTA's part_s[rank][j]
+    auto table_epilogue = [&]() {
+      if (warp != 0) return;
+      const int jl = lane < lcap ? rowj_s[lane] : -1;
+      const float rc = jl >= 0 ? lp_f[acc_s[jl] * 3 + 2] : 0.f;
+      const bool cin = jl >= 0 && tri_in_range(rc);
+      float bd = INFINITY;
+      int bR = -1;
+      for (int c0 = 0; c0 < tr_cnt; c0 += 16) {
+        uint32_t raw[16];
+        tmem_ld16(tmem + (uint32_t)c0, raw);
+#pragma unroll
+        for (int q = 0; q < 16; ++q) {
+          const int si = c0 + q;
+          if (si < tr_cnt) {
+            const int R = tr_s0 + si;
+            const float d = __fsub_rn(1.0f, __fmul_rn(__fmul_rn(__uint_as_float(raw[q]), rc), rootr_s[R]));
+            const float lb = cin ? tri_rho_lb(d, a.tri_eps_x) : 0.f;
+            if (jl >= 0) a.rtab[(size_t)(rootoff + R) * kMaxAccept + jl] = lb;
+            const uint32_t mn = __reduce_min_sync(0xffffffffu, __float_as_uint(jl >= 0 ? lb : INFINITY));
+            if (lane == 0) mr_s[R] = __uint_as_float(mn);
+            if (cin && d < bd) {
+              bd = d;
+              bR = R;
+            }
+          }
+        }
+      }
+      if (jl >= 0)
+        for (int q = 0; q < C; ++q)
+          st_cluster_v2f(map_shared(&part_s[(int)rank * kMaxAccept + jl], q),
+                         make_float2(bd, __int_as_float(bR)));
+      // the slice's minima to every other CTA, four at a time (tr_s0 is a multiple of 16)
+      __syncwarp();
+      if (lane < C && lane != (int)rank)
+        for (int si = 0; si < tr_cnt; si += 4) {
+          const U4 v = lds(&mr_s[tr_s0 + si]);
+          asm volatile("st.shared::cluster.v4.u32 [%0], {%1,%2,%3,%4};"
+                       :: "r"(map_shared(&mr_s[tr_s0 + si], lane)), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
+                       : "memory");
+        }
+    };
+    // every CTA alike: each accepted centre's nearest root over the slices that
+    // existed this round (the lowest root on ties); a centre farther than kTriTau
+    // from every root becomes a root (while the request has room), else it is
+    // attached to that root with e = rho_ub; then the new roots' rows are copied to
+    // the request's root rows (for the next rounds' tables)
+    auto tri_merge = [&](int nA, int nroot_start) {
+      if (warp == 0) {
+        float bd = INFINITY;
+        int bR = -1;
+        if (lane < nA)
+          for (int q = 0; q < C; ++q)
+            if (q * tr_w < nroot_start) {
+              const float2 pv = part_s[q * kMaxAccept + lane];
+              const int R = __float_as_int(pv.y);
+              if (R >= 0 && pv.x < bd) {
+                bd = pv.x;
+                bR = R;
+              }
+            }
+        const float rc = lane < nA ? lp_f[acc_s[lane] * 3 + 2] : 0.f;
+        const bool cin = lane < nA && tri_in_range(rc);
+        float e = INFINITY;
+        int root = -1;
+        bool want = false;
+        if (cin) {
+          if (bR < 0) {
+            want = true;
+          } else {
+            root = bR;
+            e = tri_rho_ub(bd, a.tri_eps_x);
+            want = !(e <= kTriTau);
+          }
+        }
+        const unsigned bal = __ballot_sync(0xffffffffu, want);
+        const int id = nroot + __popc(bal & ((1u << lane) - 1u));
+        const bool made = want && id < rcap;
+        if (made) {
+          root = id;
+          e = 0.f;
+          rootr_s[id] = rc;
+        }
+        if (lane < nA) {
+          croot_s[lane] = root;
+          ce_s[lane] = e;
+        }
+        const unsigned mb = __ballot_sync(0xffffffffu, made);
+        if (made) nrl_s[__popc(mb & ((1u << lane) - 1u))] = make_int2(id, lp_idx[acc_s[lane]]);
+        if (lane == 0) nrl_s[kMaxAccept] = make_int2(__popc(mb), 0);
+      }
+      __syncthreads();
+      const int nnew = nrl_s[kMaxAccept].x;
+      for (int u = (int)rank + C * warp; u < nnew; u += C * kSelectWarps) {
+        const int2 nr = nrl_s[u];
+        const char *src = xreq + (long long)nr.y * rb;
+        const int i = nr.x % kRootGroup;
+        const int nkb = tc_kblocks(dv);   // rows are padded to whole K blocks (zeros)
+        char *grp = a.roots + (long long)(rootoff + nr.x - i) * (nkb * 128) + i * 128;
+        for (int v = lane; v < nkb * 8; v += 32)   // chunk v: K block v / 8, chunk v % 8
+          *reinterpret_cast<U4 *>(grp + (v >> 3) * kRootGroupKbBytes + (((v & 7) ^ (i & 7)) << 4)) =
+              v < rb / 16 ? ldg(src + 16 * v) : U4{0, 0, 0, 0};
+      }
+      fence_proxy_async_global();   // the next rounds read these rows through TMA
+      nroot += nnew;
+    };
+
     // ---- seed (Eq. 9): one round that accepts argmax w~ ----
+    if constexpr (TC) deep_rebuild(false);
     publish(0);
     cluster_sync();
     if (threadIdx.x == 0) {
@@ -827,7 +1346,8 @@ select_kernel(const __grid_constant__ SelectArgs a) {
       stage_list(1);
       wait_rows();
       __syncthreads();
-      update(1);
+      if (tri) tri_merge(1, 0);   // the seed is the first root
+      update(1, false);
       __syncthreads();
     }
 
@@ -836,6 +1356,18 @@ select_kernel(const __grid_constant__ SelectArgs a) {
       const int par = round & 1;
       publish(par);
       cluster_sync();
+      if (tri) {
+        // this round's slice of the roots: its rows start streaming now, while the
+        // candidate list is built (every ring stage is free at a round's start).  The
+        // barrier above orders the last merge's root-row copies (any CTA) before these
+        // tensor loads.
+        tri_slice();
+        if (threadIdx.x == 64 && tr_pre > 0) {
+          fence_proxy_async_global();
+          fence_proxy_async_smem();
+          table_load(tr_pre, true);   // every slot is free at a round's start
+        }
+      }
       if (TC && early && warp > 0) {   // warps 1.. copy while warp 0 builds the list
         for (int q = 0; q < C; ++q)
           for (int e = 0; e < a.mc; ++e) {
@@ -857,60 +1389,40 @@ select_kernel(const __grid_constant__ SelectArgs a) {
                        (uint32_t)rb, bar);
           }
       }
-      // candidate list: published top-mc entries above U, best first, at most lcap
+      // candidate list: published entries above U, best first, at most lcap.  Each
+      // CTA's published entries are sorted, so the list is a C-way merge: lane q
+      // holds the head of CTA q's entries and the warp takes the largest head.
       if (warp == 0) {
         const int kPer = a.mc;
-        const int ne = C * kPer;
-        const unsigned long long u5 = lane < C ? pub_key[(par * kMaxCluster + lane) * kTopMax + kPer] : 0ull;
-        const uint32_t uhi = __reduce_max_sync(0xffffffffu, (uint32_t)(u5 >> 32));
-        const uint32_t ulo = __reduce_max_sync(0xffffffffu, (uint32_t)(u5 >> 32) == uhi ? (uint32_t)u5 : 0u);
-        const unsigned long long U = ((unsigned long long)uhi << 32) | ulo;
-        int slot0 = 0, slot1 = 0;
-        unsigned long long ke0 = 0ull, ke1 = 0ull;
-        if (lane < ne) {
-          slot0 = (par * kMaxCluster + lane / kPer) * kTopMax + lane % kPer;
-          ke0 = pub_key[slot0];
-        }
-        if (lane + 32 < ne) {
-          slot1 = (par * kMaxCluster + (lane + 32) / kPer) * kTopMax + (lane + 32) % kPer;
-          ke1 = pub_key[slot1];
-        }
-        const bool c0 = ke0 > U, c1 = ke1 > U;
-        // rank among the candidates: non-candidates are masked to 0 (below every candidate)
-        const unsigned long long m0 = c0 ? ke0 : 0ull, m1 = c1 ? ke1 : 0ull;
-        int pos0 = 0, pos1 = 0;
-#pragma unroll
-        for (int src = 0; src < 32; ++src) {
-          const unsigned long long a0 = shfl_u64(m0, src), a1 = shfl_u64(m1, src);
-          pos0 += (a0 > ke0 ? 1 : 0) + (a1 > ke0 ? 1 : 0);
-          pos1 += (a0 > ke1 ? 1 : 0) + (a1 > ke1 ? 1 : 0);
-        }
+        const int base = (par * kMaxCluster + lane) * kTopMax;
+        const unsigned long long u5 = lane < C ? pub_key[base + kPer] : 0ull;
+        const unsigned long long U = warp_max_u64(u5);
+        int ptr = 0, n = 0;
+        unsigned long long head = (lane < C && kPer > 0) ? pub_key[base] : 0ull;
         unsigned long long cut = 0ull;
-        auto place = [&](bool cand, int pos, unsigned long long ke, int slot) {
-          if (!cand) return;
-          if (pos < lcap) {
-            const float4 f = pub_f[slot];
-            lp_key[pos] = ke;
-            lp_idx[pos] = key_index(ke);
-            lp_row[pos] = (slot % kTopMax) + (slot / kTopMax - par * kMaxCluster) * a.mc;
-            lp_f[pos * 3 + 0] = f.x;
-            lp_f[pos * 3 + 1] = f.y;
-            lp_f[pos * 3 + 2] = f.z;
-          } else if (pos == lcap) {
-            cut = ke;
+        while (true) {
+          const unsigned long long best = warp_max_u64(head);
+          if (best <= U) break;            // also the end of every list (key 0)
+          if (n == lcap) {
+            cut = best;                    // the first candidate the list cannot hold
+            break;
           }
-        };
-        place(c0, pos0, ke0, slot0);
-        place(c1, pos1, ke1, slot1);
-        const int ncand = __popc(__ballot_sync(0xffffffffu, c0)) + __popc(__ballot_sync(0xffffffffu, c1));
-        {
-          const uint32_t chi = __reduce_max_sync(0xffffffffu, (uint32_t)(cut >> 32));
-          const uint32_t clo = __reduce_max_sync(0xffffffffu, (uint32_t)(cut >> 32) == chi ? (uint32_t)cut : 0u);
-          cut = ((unsigned long long)chi << 32) | clo;
+          if (head == best) {              // keys are unique: one lane
+            const float4 f = pub_f[base + ptr];
+            lp_key[n] = best;
+            lp_idx[n] = key_index(best);
+            lp_row[n] = ptr + lane * kPer;  // the early copy's row of this entry
+            lp_f[n * 3 + 0] = f.x;
+            lp_f[n * 3 + 1] = f.y;
+            lp_f[n * 3 + 2] = f.z;
+            ++ptr;
+            head = ptr < kPer ? pub_key[base + ptr] : 0ull;
+          }
+          ++n;
         }
         if (lane == 0) {
           misc[0] = cut > U ? cut : U;               // U' bounds everything outside L
-          misc[1] = (unsigned long long)min(ncand, lcap);
+          misc[1] = (unsigned long long)n;
         }
       }
       __syncthreads();
@@ -949,6 +1461,7 @@ select_kernel(const __grid_constant__ SelectArgs a) {
                           (kb >= kGramChains || k != 0) ? 1u : 0u);
             umma_commit(tpair);
           }
+          table_poll();   // root-table stages that have landed
           __syncwarp();
           twait(tpair, tc_pph);
           tc_pph ^= 1u;
@@ -1050,8 +1563,12 @@ select_kernel(const __grid_constant__ SelectArgs a) {
           }
         }
       }
+      table_poll();
       cluster_sync();
-      // replay the greedy on L (warp 0; lane u holds member u)
+      // replay the greedy on L (warp 0; lane u holds member u); meanwhile the root
+      // table's service threads finish its copies and MMAs
+      if (tri && tr_nts > 0 && threadIdx.x == 32) table_mma(true);
+      else if (tri && tr_nts > 0 && threadIdx.x == 64) table_load(tr_nts, true);
       if (warp == 0) {
         const unsigned long long Up = misc[0];
         bool pending = lane < nL;
@@ -1094,8 +1611,35 @@ select_kernel(const __grid_constant__ SelectArgs a) {
       taken += nA;
       __syncthreads();
       if (taken < K) {
-        update(nA);
+        const int nroot_start = nroot;
+        if (tri) {
+          if (warp == 0) {   // cbuf row -> accepted slot
+            if (lane < kLcap) rowj_s[lane] = -1;
+            __syncwarp();
+            if (lane < nA) rowj_s[lp_row[acc_s[lane]]] = lane;
+          }
+          if (tr_nts > 0) {
+            __syncthreads();   // the service threads finished their part during the replay
+            twait(ttab, tc_tph);
+            tc_tph ^= 1u;
+            tc_fence_after();
+          }
+          __syncthreads();
+          if (tr_cnt > 0) table_epilogue();
+          tc_fence_before();
+          cluster_sync();
+          tc_fence_after();
+          tri_merge(nA, nroot_start);
+        }
+        update(nA, tri && nroot_start > 0);
         __syncthreads();
+      } else if (tri && tr_nts > 0) {
+        // the selection ended this round: the table's copies and MMAs still complete
+        // (nothing may be in flight when the CTA exits)
+        __syncthreads();
+        twait(ttab, tc_tph);
+        tc_tph ^= 1u;
+        tc_fence_after();
       }
     }
     if constexpr (TC) {

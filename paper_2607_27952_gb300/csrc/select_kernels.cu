@@ -118,13 +118,13 @@ EncodeTiledFn encode_tiled() {
   return fn;
 }
 
-// X as a [total_vis][dv] bf16 tensor, 64 x 128 boxes, 128-byte swizzle.
-bool encode_x_map(CUtensorMap *m, const void *x, long long rows, int dv) {
+// X as a [rows][dv] bf16 tensor, 64-element x box_rows boxes, 128-byte swizzle.
+bool encode_x_map(CUtensorMap *m, const void *x, long long rows, int dv, int box_rows = kTcBM) {
   EncodeTiledFn fn = encode_tiled();
   if (fn == nullptr || rows <= 0) return false;
   cuuint64_t dims[2] = {(cuuint64_t)dv, (cuuint64_t)rows};
   cuuint64_t strides[1] = {(cuuint64_t)dv * 2};
-  cuuint32_t box[2] = {(cuuint32_t)kTcBK, (cuuint32_t)kTcBM};
+  cuuint32_t box[2] = {(cuuint32_t)kTcBK, (cuuint32_t)box_rows};
   cuuint32_t estr[2] = {1, 1};
   return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(x), dims, strides, box, estr,
             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -191,7 +191,7 @@ cudaError_t launch_select(const Plan &pl, const float *w, const void *x, int32_t
   // When no cluster size fits the tensor-core update (its accumulators take a
   // TMEM column per list entry and 128-row tile, so very long requests do not
   // fit), the sizes are costed again for the CUDA-core update.
-  int C = 0, tpc = 0, cache_rows = 0, ring = 0, lcap = kLcap / 2, stages = 0, kps = 1;
+  int C = 0, tpc = 0, cache_rows = 0, ring = 0, lcap = kLcap / 2, stages = 0, kps = 1, roots = 0;
   size_t smem = 0;
   double best = 0.0;
   void *fn = nullptr;
@@ -204,7 +204,7 @@ cudaError_t launch_select(const Plan &pl, const float *w, const void *x, int32_t
     const int tpc_c = (pl.max_vis + c - 1) / c;
     const int tb_c = select_tb(pl.elem, tc, tpc_c);
     void *fn_c = pick_select(pl.dtype, nch, tb_c, tc);
-    int cache_c = 0, ring_c = 0, lcap_c = 0, stages_c = 0, kps_c = 1;
+    int cache_c = 0, ring_c = 0, lcap_c = 0, stages_c = 0, kps_c = 1, roots_c = 0;
     size_t smem_c = 0;
     if (tc) {
       // the list length is the MMA N: lcap accumulator columns per 128-row tile; the
@@ -212,7 +212,12 @@ cudaError_t launch_select(const Plan &pl, const float *w, const void *x, int32_t
       const int tiles = (tpc_c + kTcBM - 1) / kTcBM;
       // stages of kps boxes: the largest kps (<= 4) that still leaves 2 stages
       for (int lc = (c <= 4 ? kLcap : kLcap / 2); lc >= kLcap / 2 && lcap_c == 0; lc /= 2) {
-        const size_t fixed = select_smem(0, rb, tpc_c, 0, tb_c, pl.elem, lc, 1, 0).total;
+        // Row skipping: a CTA's slice of the roots takes TMEM columns of the tile
+        // accumulators (at most 128, whole groups of 16), so the request's roots are
+        // capped at that slice times the cluster size.
+        const int s_cap = std::min(128, tiles * lc / kRootGroup * kRootGroup);
+        const int roots_lc = (pl.root_rows > 0 && s_cap >= kRootGroup) ? std::min(kMaxRoots, s_cap * c) : 0;
+        const size_t fixed = select_smem(0, rb, tpc_c, 0, tb_c, pl.elem, lc, 1, 0, 1, roots_lc).total;
         // TMEM: lc columns per tile plus kGramChains x lc for the list's Gram
         if (fixed + 2 * (size_t)kTcBoxBytes > (size_t)di.optin ||
             (tiles + kGramChains) * lc > kTmemCols)
@@ -223,7 +228,8 @@ cudaError_t launch_select(const Plan &pl, const float *w, const void *x, int32_t
         kps_c = std::min(kps_c, tc_kblocks(pl.dv));
         stages_c = (int)std::min<size_t>(kTcMaxStages, room / ((size_t)kps_c * kTcBoxBytes));
         lcap_c = lc;
-        smem_c = select_smem(0, rb, tpc_c, 0, tb_c, pl.elem, lc, 1, stages_c, kps_c).total;
+        roots_c = roots_lc;
+        smem_c = select_smem(0, rb, tpc_c, 0, tb_c, pl.elem, lc, 1, stages_c, kps_c, roots_c).total;
       }
       if (lcap_c == 0) continue;
     } else {
@@ -266,7 +272,7 @@ cudaError_t launch_select(const Plan &pl, const float *w, const void *x, int32_t
     const double cost = waves * round_cycles;
     if (C == 0 || cost < best) {
       best = cost; C = c; tpc = tpc_c; cache_rows = cache_c; smem = smem_c; ring = ring_c;
-      lcap = lcap_c; fn = fn_c; stages = stages_c; kps = kps_c;
+      lcap = lcap_c; fn = fn_c; stages = stages_c; kps = kps_c; roots = roots_c;
     }
   }
   }
@@ -280,12 +286,13 @@ cudaError_t launch_select(const Plan &pl, const float *w, const void *x, int32_t
   a.meta = reinterpret_cast<const int32_t *>(ws + pl.off_meta);
   a.order = reinterpret_cast<const int32_t *>(ws + pl.off_order);
   a.dv = pl.dv; a.row_bytes = rb; a.tpc_max = tpc; a.cache_rows = cache_rows; a.csize = C;
-  // Candidates each CTA publishes: enough that the list approximates the global
-  // top picks, at most 64 in all (the list is built by one warp, two per lane).
-  // The tensor-core update ranks 16 per CTA and accepts up to 32 picks a round;
-  // the CUDA-core update ranks 8 and accepts 16 (its register blocking).
+  // Candidates each CTA publishes (the cluster's list is a C-way merge of the
+  // published lists, so its cost does not grow with them).  The tensor-core variant
+  // publishes its top 16 (its incremental candidate list holds them cheaply) and
+  // accepts up to 32 picks a round; the CUDA-core update ranks 8 (4 in clusters of
+  // more than 4 CTAs) and accepts 16 (its register blocking).
   if (tc) {
-    a.mc = std::min(16, 64 / C);
+    a.mc = kTopMax - 1;   // the candidate list keeps every CTA's top keys cheaply
     a.max_accept = kMaxAccept;
   } else {
     a.mc = C <= 4 ? 8 : 4;
@@ -302,6 +309,14 @@ cudaError_t launch_select(const Plan &pl, const float *w, const void *x, int32_t
     a.tc_stages = stages;
     a.tc_kps = kps;
     a.tc_eps = tc_distance_eps(pl.dv);
+    // row skipping (the root capacity was chosen with the shared-memory plan)
+    if (roots > 0) {
+      a.tri = 1;
+      a.root_cap = roots;
+      a.roots = ws + pl.off_roots;
+      a.rtab = reinterpret_cast<float *>(ws + pl.off_rtab);
+      a.tri_eps_x = a.tc_eps + kTriEpsC;
+    }
   }
 
   cudaLaunchConfig_t cfg = {};

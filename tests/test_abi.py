@@ -167,7 +167,18 @@ def test_scores_rows_workspace_grows_with_rows(lib):
     many = last.last_scores_rows_workspace_size(prob, last.QueryRows([0, 3, 6], [6, 7, 9, 10, 15, 19]))
     assert many > one > 0
     # one row per request runs the last-row kernels: the workspace holds their plan
-    assert one >= last.last_workspace_size(prob)
+    # (the scoring part of last_workspace_size: with no budgets the selection's
+    # root-row scratch is empty)
+    assert one >= last.last_workspace_size(_problem(cu_keep=[0, 0, 0]))
+
+
+def test_workspace_holds_selection_root_rows(lib):
+    """bf16 problems carry the greedy's root rows: min(k_b, 1024) feature rows and a
+    32-column bound table per request, on top of the scoring scratch."""
+    base = last.last_workspace_size(_problem(cu_keep=[0, 0, 0]))
+    full = last.last_workspace_size(_problem())
+    assert full - base >= 5 * (256 * 2 + 32 * 4)
+    assert last.last_workspace_size(_problem(dtype="f32")) < full + 4096
 
 
 def test_workspace_checks(lib):

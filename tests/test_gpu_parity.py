@@ -248,3 +248,25 @@ def test_full_size_video(pct):
     for b in range(wl.batch):
         big = idx[wl.cu_keep[b]:wl.cu_keep[b + 1]]
         assert np.isin(idx_small[small[b]:small[b + 1]], big).all(), f"request {b}: not a prefix"
+
+
+def test_gather_wide_rows():
+    """Eq. 12 has no width limit: a 4096-wide bf16 gather (twice the selection's
+    feature-width limit) is a bitwise copy of the oracle's gather."""
+    import torch
+    import paper_2607_27952_gb300 as last
+    from gpu_util import problem_of, to_dev, to_host_bits
+    wl = custom(name="gather4096", seed=71, batch=2, n_vis=[40, 75], n_text=[1, 1],
+                feat_dim=4096, dtype="bf16", keep=[9, 20])
+    prob = problem_of(wl)
+    dev = torch.device("cuda:0")
+    rng = np.random.default_rng(3)
+    idx = np.concatenate([np.sort(rng.choice(40, 9, replace=False)),
+                          np.sort(rng.choice(75, 20, replace=False))]).astype(np.int32)
+    out = torch.zeros((29, 4096), dtype=torch.bfloat16, device=dev)
+    ws = last.workspace(prob, dev)
+    last.last_gather(prob, to_dev(wl.x, dev), torch.from_numpy(idx).to(dev), out, ws)
+    last.last_poll(ws)
+    got = to_host_bits(out)
+    assert np.array_equal(got[:9], oracle.gather(wl.x[:40], idx[:9]))
+    assert np.array_equal(got[9:], oracle.gather(wl.x[40:115], idx[9:]))
