@@ -90,9 +90,9 @@ constexpr int kRootGroup = 16;                     // roots per group: the table
 // of the group at kb * 2048, row i at i * 128, 16-byte chunk c at (c ^ (i % 8)) * 16
 // (K-major, 128-byte swizzle).  One bulk copy then moves any run of K blocks.
 constexpr int kRootGroupKbBytes = kRootGroup * 128;
-// The root table streams through the update's ring, cut into kTabSt stages with
-// barriers of their own (the update's stages are idle while it runs), so that
-// many small bulk copies are in flight while the candidate list is processed.
+// The root table streams through the update's ring (idle while it runs) in slots
+// of one K block of 128 root rows, at most kTabSt of them, with barriers of their
+// own, so that its copies are in flight while the candidate list is processed.
 constexpr int kTabSt = 8;
 constexpr float kTriTau = 0.5f;                    // chordal radius that makes a centre a root
 // |canonical fp32 distance - exact distance| for rows of norm in [2^-50, 2^50] and
@@ -131,7 +131,7 @@ struct SelectArgs {
 struct SelectSmem {
   size_t aring, xcache, cbuf, ring, blk, w, r, dl, list, sel, wtop, pub_key, pub_f, lp_key,
       lp_f, lp_idx, lp_row, pair, acc, misc, bar, cnt, tbar, tslot, fidx, fmask, fcnt, gram, plist,
-      oroot, oe, mr, rootr, part, croot, ce, rowj, nrl, deep, total;
+      oroot, oe, mr, rootr, part, croot, ce, rowj, nrl, hard, deep, total;
 };
 // K blocks of kTcBK elements covering a feature row.
 __host__ __device__ inline int tc_kblocks(int dv) { return (dv + kTcBK - 1) / kTcBK; }
@@ -184,7 +184,8 @@ __host__ __device__ inline SelectSmem select_smem(int cache_rows, int row_bytes,
   s.bar = o; o += sizeof(unsigned long long);
   s.cnt = o; o += sizeof(int) * kMaxCluster;
   o = align16(o);
-  s.tbar = o; o += tc ? sizeof(unsigned long long) * (2 * kTcMaxStages + 4 + 2 * kTabSt) : 0;
+  s.tbar = o; o += tc ? sizeof(unsigned long long) * (2 * kTcMaxStages + 3 + 2 * kTabSt) : 0;
+  o = align16(o);   // later regions take 16-byte vector accesses (mr: v4 loads and cluster stores)
   s.tslot = o; o += tc ? 16 : 0;
   s.fidx = o; o += tc ? align16(sizeof(int) * tpc_max) : 0;
   s.fmask = o; o += tc ? align16(sizeof(uint32_t) * tpc_max) : 0;
@@ -205,6 +206,7 @@ __host__ __device__ inline SelectSmem select_smem(int cache_rows, int row_bytes,
   s.ce = o; o += tri ? sizeof(float) * kMaxAccept : 0;
   s.rowj = o; o += tri ? sizeof(int) * kLcap : 0;
   s.nrl = o; o += tri ? sizeof(int2) * (kMaxAccept + 1) : 0;
+  s.hard = o; o += tri ? sizeof(int2) * kMaxCluster : 0;   // every CTA's (hard, live) counts
   s.deep = o; o += tc ? sizeof(unsigned long long) * kDeep + 16 : 0;   // candidate list + flag
   s.total = align16(o) + 1024;   // slack for aligning the base to 1024 bytes
   return s;
@@ -402,10 +404,8 @@ select_kernel(const __grid_constant__ SelectArgs a) {
   unsigned long long *tdone = tempty + kTcMaxStages;
   unsigned long long *tpair = tdone + 1;
   unsigned long long *ttab = tpair + 1;   // the round's root table is in TMEM
-  unsigned long long *txb = ttab + 1;     // rows of the exact step (bulk copies)
-  unsigned long long *tbf = txb + 1;      // root-table stages: landed
+  unsigned long long *tbf = ttab + 1;     // root-table stages: landed
   unsigned long long *tbe = tbf + kTabSt; // root-table stages: consumed by the MMAs
-  uint32_t txph = 0;
   if (threadIdx.x == 0) {
     mbar_init(bar, 1);
     if constexpr (TC) {
@@ -416,7 +416,6 @@ select_kernel(const __grid_constant__ SelectArgs a) {
       mbar_init(tdone, 1);
       mbar_init(tpair, 1);
       mbar_init(ttab, 1);
-      mbar_init(txb, 1);
       for (int i = 0; i < kTabSt; ++i) {
         mbar_init(&tbf[i], 1);
         mbar_init(&tbe[i], 1);
@@ -1024,10 +1023,10 @@ select_kernel(const __grid_constant__ SelectArgs a) {
       tc_fence_before();
       __syncthreads();
       }   // dense
-      // 4. exact canonical distances for the flagged pairs.  The flagged tokens' rows
-      //    are bulk-copied into the ring (idle now) in batches, every copy of a batch
-      //    in flight at once; then a warp per token evaluates its pairs from shared
-      //    memory in the canonical order.
+      // 4. exact canonical distances for the flagged pairs.  A warp per flagged token
+      //    reads the token's row straight from global memory (the next token's row is
+      //    in flight while the current one is evaluated) and evaluates its pairs in the
+      //    canonical order against the centre rows in shared memory.
       const int nf = *fcnt;
       auto exact_token = [&](int t, unsigned msk, const U4 *xv) {
         const float ri = r_s[t];
@@ -1065,29 +1064,29 @@ select_kernel(const __grid_constant__ SelectArgs a) {
           }
         }
       };
-      const int per_batch = min(nstage * a.tc_kps * kTcBoxBytes / rb, 64);
-      for (int b0 = 0; b0 < nf; b0 += per_batch) {
-        const int nb = min(per_batch, nf - b0);
-        if (threadIdx.x == 0) {
-          fence_proxy_async_smem();   // the last batch's reads precede these writes
-          mbar_expect_tx(txb, (uint32_t)(nb * rb));
-          for (int i = 0; i < nb; ++i)
-            bulk_g2s(aring + (long long)i * rb, xg + (long long)fidx[b0 + i] * rb, (uint32_t)rb, txb);
-        }
-        mbar_wait_bounded(txb, txph, a.err, kErrTimeout);
-        txph ^= 1u;
-        for (int f = b0 + warp; f < b0 + nb; f += kSelectWarps) {
-          const uint32_t row = smem_addr(aring + (long long)(f - b0) * rb);
-          U4 xv[NCH];
+      auto load_row = [&](int t, U4 *xv) {
+        const char *row = xg + (long long)t * rb;
 #pragma unroll
-          for (int g = 0; g < NCH; ++g) {
-            const int col = 256 * g + 8 * lane;
-            xv[g] = col < dv ? lds32(row + (uint32_t)(col * 2)) : U4{0, 0, 0, 0};
-          }
-          exact_token(fidx[f], fmask[f], xv);
+        for (int g = 0; g < NCH; ++g) {
+          const int col = 256 * g + 8 * lane;
+          xv[g] = col < dv ? ldg_stream(row + col * 2) : U4{0, 0, 0, 0};
         }
-        __syncthreads();
+      };
+      {
+        U4 xa[NCH], xb[NCH];
+        int f = warp;
+        if (f < nf) load_row(fidx[f], xa);
+        while (f < nf) {
+          if (f + kSelectWarps < nf) load_row(fidx[f + kSelectWarps], xb);
+          exact_token(fidx[f], fmask[f], xa);
+          f += kSelectWarps;
+          if (f >= nf) break;
+          if (f + kSelectWarps < nf) load_row(fidx[f + kSelectWarps], xa);
+          exact_token(fidx[f], fmask[f], xb);
+          f += kSelectWarps;
+        }
       }
+      __syncthreads();
       // 5. the candidate list from the new deltas; all tokens are re-ranked only when
       //    too few of its entries are still known to lead
       deep_refresh();
@@ -1131,72 +1130,82 @@ select_kernel(const __grid_constant__ SelectArgs a) {
 
     // ---- triangle-inequality bookkeeping (tensor-core variant) ----
     // Each round the cluster's CTAs split the request's roots: CTA `rank` takes roots
-    // [tr_s0, tr_s0 + tr_cnt) and forms their dot products with every list row on the
-    // tensor cores (A = the list rows in cbuf, B = the roots' rows streamed through
-    // the ring by bulk copies, tr_kbps K blocks of one group per ring stage; fp32
-    // accumulators in TMEM columns [0, tr_w), which the update's tiles reuse later).
-    int tr_s0 = 0, tr_cnt = 0, tr_w = 0, tr_kbps = 1, tr_nts = 0, tr_pre = 0;
+    // [tr_s0, tr_s0 + tr_cnt) (at most 128) and forms their dot products with every
+    // list row on the tensor cores: A = the slice's root rows (M = 128, one TMEM lane
+    // per root), B = the list rows in cbuf (N = lcap), fp32 accumulators in TMEM
+    // columns [0, lcap), which the update's first tile reuses later.  The root rows
+    // stream through the ring one K block per stage: the slice's groups of 16 rows
+    // land side by side, so a stage is the K-major 128-byte-swizzled image of up to
+    // 128 rows (rows past the slice hold stale data and only reach unused lanes).
+    int tr_s0 = 0, tr_cnt = 0, tr_w = 0, tr_ngrp = 0, tr_nts = 0, tr_pre = 0;
+    int tab_slots = 2, tab_stride = 0;   // stage slots and their spacing
     int tr_issued = 0, tr_mma = 0;   // thread 64: stages issued; thread 32: stages consumed
-    uint32_t tb_pit = 0, tb_mit = 0;  // their running stage counters (barrier phases)
+    // Per-slot barrier phases (the slot count changes from round to round): thread 64
+    // keeps the parity of each slot's fills so far and which slots were ever filled,
+    // thread 32 the parity of each slot's consumptions so far.
+    uint32_t tb_fpar = 0, tb_fused = 0, tb_cpar = 0;
     uint32_t tc_tph = 0;   // root-table phase
-    const int tab_sb = (nstage * a.tc_kps * kTcBoxBytes / kTabSt) / kRootGroupKbBytes * kRootGroupKbBytes;
+    constexpr int kTabSlot = kTcBM * 128;   // one K block of 128 root rows
+    const int tab_ring = nstage * a.tc_kps * kTcBoxBytes;
     auto tri_slice = [&]() {
       const int per = ((nroot + C - 1) / C + kRootGroup - 1) / kRootGroup * kRootGroup;
       tr_s0 = min(nroot, (int)rank * per);
       tr_cnt = min(nroot, tr_s0 + per) - tr_s0;
       tr_w = per;
-      tr_kbps = tab_sb / kRootGroupKbBytes;   // K blocks of one group per stage
-      const int ngrp = (tr_cnt + kRootGroup - 1) / kRootGroup;
-      tr_nts = ngrp * ((tc_kblocks(dv) + tr_kbps - 1) / tr_kbps);
-      tr_pre = min(tr_nts, kTabSt);
+      tr_ngrp = (tr_cnt + kRootGroup - 1) / kRootGroup;
+      tr_nts = tr_cnt > 0 ? tc_kblocks(dv) : 0;
+      tab_stride = kTabSlot;
+      tab_slots = min(kTabSt, tab_ring / kTabSlot);
+      tr_pre = min(tr_nts, tab_slots);
       tr_issued = 0;
       tr_mma = 0;
     };
     // thread 64: bulk copies of table stages [tr_issued, upto) into the ring; stage s
-    // holds K blocks [kb0, kb0 + tr_kbps) of root group s / (stages per group).  A
-    // stage slot is reused once the MMAs of its previous stage are done; `block`
-    // false issues only what is free now.
+    // is K block s of every group of the slice.  A stage slot is reused once the MMAs
+    // of its previous stage are done; `block` false issues only what is free now.
     auto table_load = [&](int upto, bool block) {
       char *aring = reinterpret_cast<char *>(smem + S.aring);
       const int nkb = tc_kblocks(dv);
-      const int spg = (nkb + tr_kbps - 1) / tr_kbps;
-      for (; tr_issued < upto; ++tr_issued, ++tb_pit) {
-        const int st = tb_pit % kTabSt;
-        if (tb_pit >= (uint32_t)kTabSt) {
-          const uint32_t par = ((tb_pit / kTabSt) - 1) & 1;
+      for (; tr_issued < upto; ++tr_issued) {
+        const int st = tr_issued % tab_slots;
+        if ((tb_fused >> st) & 1u) {   // the slot's previous fill must have been consumed
+          const uint32_t par = ((tb_fpar >> st) & 1u) ^ 1u;
           if (!block && !mbar_try_wait(&tbe[st], par)) break;
-          if (block && !twait(&tbe[st], par)) continue;
+          if (block && !twait(&tbe[st], par)) {
+            tb_fpar ^= 1u << st;   // the stage is skipped: the call reports the timeout
+            continue;
+          }
         }
-        const int g = tr_issued / spg, kb0 = (tr_issued % spg) * tr_kbps, nb = min(tr_kbps, nkb - kb0);
-        const char *src = a.roots + (long long)(rootoff + tr_s0 + g * kRootGroup) * (nkb * 128) +
-                          (long long)kb0 * kRootGroupKbBytes;
-        mbar_expect_tx(&tbf[st], (uint32_t)(nb * kRootGroupKbBytes));
-        bulk_g2s(aring + st * tab_sb, src, (uint32_t)(nb * kRootGroupKbBytes), &tbf[st]);
+        tb_fpar ^= 1u << st;
+        tb_fused |= 1u << st;
+        const char *src = a.roots + (long long)(rootoff + tr_s0) * (nkb * 128) +
+                          (long long)tr_issued * kRootGroupKbBytes;
+        mbar_expect_tx(&tbf[st], (uint32_t)(tr_ngrp * kRootGroupKbBytes));
+        for (int g = 0; g < tr_ngrp; ++g)
+          bulk_g2s(aring + st * tab_stride + g * kRootGroupKbBytes,
+                   src + (long long)g * nkb * kRootGroupKbBytes, (uint32_t)kRootGroupKbBytes, &tbf[st]);
       }
     };
-    // thread 32: the table's MMAs (N = 16 roots of one group into TMEM columns
-    // [16 g, 16 g + 16)) for stages that have landed; `block` waits for all of them
-    // and then commits to ttab
+    // thread 32: the table's MMAs (M = 128 root lanes, N = lcap list rows, one K
+    // block per stage) for stages that have landed; `block` waits for all of them and
+    // then commits to ttab
     auto table_mma = [&](bool block) {
-      const int nkb = tc_kblocks(dv);
-      const int spg = (nkb + tr_kbps - 1) / tr_kbps;
       const uint32_t aring_sa = smem_addr(smem + S.aring);
-      const uint32_t idesc = umma_idesc_bf16(kTcBM, kRootGroup);
-      for (; tr_mma < tr_nts; ++tr_mma, ++tb_mit) {
-        const int st = tb_mit % kTabSt;
-        const uint32_t par = (tb_mit / kTabSt) & 1;
+      const uint32_t idesc = umma_idesc_bf16(kTcBM, lcap);
+      for (; tr_mma < tr_nts; ++tr_mma) {
+        const int st = tr_mma % tab_slots;
+        const uint32_t par = (tb_cpar >> st) & 1u;
         if (!block && !mbar_try_wait(&tbf[st], par)) return;
         const bool ok = !block || twait(&tbf[st], par);
+        tb_cpar ^= 1u << st;
         tc_fence_after();
         if (ok) {
-          const int g = tr_mma / spg, kb0 = (tr_mma % spg) * tr_kbps, nb = min(tr_kbps, nkb - kb0);
-          for (int q = 0; q < nb; ++q)
+          const int kb = tr_mma;
 #pragma unroll
-            for (int k = 0; k < kTcBK / 16; ++k)
-              umma_bf16(tmem + (uint32_t)(g * kRootGroup),
-                        umma_desc_sw128(cbuf_sa + (kb0 + q) * lcap * 128 + k * 32),
-                        umma_desc_sw128(aring_sa + st * tab_sb + q * kRootGroupKbBytes + k * 32),
-                        idesc, ((kb0 + q) | k) != 0 ? 1u : 0u);
+          for (int k = 0; k < kTcBK / 16; ++k)
+            umma_bf16(tmem, umma_desc_sw128(aring_sa + st * tab_stride + k * 32),
+                      umma_desc_sw128(cbuf_sa + kb * lcap * 128 + k * 32), idesc,
+                      (kb | k) != 0 ? 1u : 0u);
         }
         umma_commit(&tbe[st]);
       }
@@ -1208,50 +1217,69 @@ select_kernel(const __grid_constant__ SelectArgs a) {
       if (threadIdx.x == 32) table_mma(false);
       else if (threadIdx.x == 64) table_load(tr_nts, false);
     };
-    // warp 0 (TMEM lanes = cbuf rows): for every root of the slice, the lower bound
-    // rho_lb(R, c_j) per accepted centre into the global table, their minimum over
-    // the centres into every CTA's mr_s[R], and per centre the nearest root of the
-    // slice into every CTA's part_s[rank][j]
+    // warps 0-3 (TMEM lane = root of the slice): for the thread's root, the lower
+    // bound rho_lb(R, c_j) per accepted centre into the global table and their minimum
+    // into every CTA's mr_s[R]; per accepted centre, the nearest root of the slice
+    // (the lowest root on ties) into every CTA's part_s[rank][j]
     auto table_epilogue = [&]() {
-      if (warp != 0) return;
-      const int jl = lane < lcap ? rowj_s[lane] : -1;
-      const float rc = jl >= 0 ? lp_f[acc_s[jl] * 3 + 2] : 0.f;
-      const bool cin = jl >= 0 && tri_in_range(rc);
-      float bd = INFINITY;
-      int bR = -1;
-      for (int c0 = 0; c0 < tr_cnt; c0 += 16) {
+      if (warp >= 4) return;
+      unsigned long long *near = wtop;   // [4 warps][kMaxAccept] (idle until the update)
+      const int si = 32 * warp + lane;
+      const bool valid = si < tr_cnt;
+      const int R = tr_s0 + si;
+      const float rr = valid ? rootr_s[R] : 0.f;
+      float *trow = a.rtab + (size_t)(rootoff + (valid ? R : tr_s0)) * kMaxAccept;
+      float mn = INFINITY;
+      for (int c0 = 0; c0 < lcap; c0 += 16) {
         uint32_t raw[16];
-        tmem_ld16(tmem + (uint32_t)c0, raw);
+        tmem_ld16(tmem + ((uint32_t)(32 * warp) << 16) + (uint32_t)c0, raw);
 #pragma unroll
         for (int q = 0; q < 16; ++q) {
-          const int si = c0 + q;
-          if (si < tr_cnt) {
-            const int R = tr_s0 + si;
-            const float d = __fsub_rn(1.0f, __fmul_rn(__fmul_rn(__uint_as_float(raw[q]), rc), rootr_s[R]));
+          const int jl = rowj_s[c0 + q];   // the same for every thread
+          if (jl >= 0) {
+            const float rc = lp_f[acc_s[jl] * 3 + 2];
+            const bool cin = tri_in_range(rc);
+            const float d = __fsub_rn(1.0f, __fmul_rn(__fmul_rn(__uint_as_float(raw[q]), rc), rr));
             const float lb = cin ? tri_rho_lb(d, a.tri_eps_x) : 0.f;
-            if (jl >= 0) a.rtab[(size_t)(rootoff + R) * kMaxAccept + jl] = lb;
-            const uint32_t mn = __reduce_min_sync(0xffffffffu, __float_as_uint(jl >= 0 ? lb : INFINITY));
-            if (lane == 0) mr_s[R] = __uint_as_float(mn);
-            if (cin && d < bd) {
-              bd = d;
-              bR = R;
+            if (valid) {
+              trow[jl] = lb;
+              mn = fminf(mn, lb);
             }
+            // (d, R) as one ordered key; NaN and invalid lanes never win
+            const uint32_t dk = (valid && cin && d == d) ? (__float_as_uint(d) ^
+                                ((__float_as_uint(d) & 0x80000000u) ? 0xffffffffu : 0x80000000u))
+                                                          : 0xffffffffu;
+            const uint32_t hk = __reduce_min_sync(0xffffffffu, dk);
+            const uint32_t rk = __reduce_min_sync(0xffffffffu, dk == hk ? (uint32_t)R : 0xffffffffu);
+            if (lane == 0) near[warp * kMaxAccept + jl] = ((unsigned long long)hk << 32) | rk;
           }
         }
       }
-      if (jl >= 0)
-        for (int q = 0; q < C; ++q)
-          st_cluster_v2f(map_shared(&part_s[(int)rank * kMaxAccept + jl], q),
-                         make_float2(bd, __int_as_float(bR)));
-      // the slice's minima to every other CTA, four at a time (tr_s0 is a multiple of 16)
-      __syncwarp();
-      if (lane < C && lane != (int)rank)
-        for (int si = 0; si < tr_cnt; si += 4) {
-          const U4 v = lds(&mr_s[tr_s0 + si]);
-          asm volatile("st.shared::cluster.v4.u32 [%0], {%1,%2,%3,%4};"
-                       :: "r"(map_shared(&mr_s[tr_s0 + si], lane)), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
-                       : "memory");
+      if (valid) mr_s[R] = mn;
+      asm volatile("bar.sync 1, 128;" ::: "memory");   // warps 0-3
+      if (warp == 0) {
+        const int jl = lane < lcap ? rowj_s[lane] : -1;
+        if (jl >= 0) {
+          unsigned long long best = near[jl];
+#pragma unroll
+          for (int w = 1; w < 4; ++w) best = min(best, near[w * kMaxAccept + jl]);
+          const uint32_t hk = (uint32_t)(best >> 32);
+          const bool any = hk != 0xffffffffu;
+          const float bd = any ? __uint_as_float(hk ^ ((hk & 0x80000000u) ? 0x80000000u : 0xffffffffu))
+                               : INFINITY;
+          const int bR = any ? (int)(uint32_t)best : -1;
+          for (int q = 0; q < C; ++q)
+            st_cluster_v2f(map_shared(&part_s[(int)rank * kMaxAccept + jl], q), make_float2(bd, __int_as_float(bR)));
         }
+        // the slice's minima to every other CTA, four at a time (tr_s0 is a multiple of 16)
+        if (lane < C && lane != (int)rank)
+          for (int s4 = 0; s4 < tr_cnt; s4 += 4) {
+            const U4 v = lds(&mr_s[tr_s0 + s4]);
+            asm volatile("st.shared::cluster.v4.u32 [%0], {%1,%2,%3,%4};"
+                         :: "r"(map_shared(&mr_s[tr_s0 + s4], lane)), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
+                         : "memory");
+          }
+      }
     };
     // every CTA alike: each accepted centre's nearest root over the slices that
     // existed this round (the lowest root on ties); a centre farther than kTriTau
@@ -1318,6 +1346,44 @@ select_kernel(const __grid_constant__ SelectArgs a) {
       nroot += nnew;
     };
 
+    // After an update: this CTA's live tokens and how many of them are "hard" (no
+    // centre near enough for a root bound to exclude any new centre: no root, a row
+    // outside the safe norm range, or 2 rho_up + e above 2), sent to every CTA.  A
+    // round whose live tokens are mostly hard skips the root table: its update
+    // streams every row anyway, and its accepted centres simply become roots.
+    int2 *hard_s = reinterpret_cast<int2 *>(smem + S.hard);
+    auto tri_count = [&]() {
+      int nh = 0, nl = 0;
+      for (int t = threadIdx.x; t < nloc; t += kSelThreads) {
+        if (!sel_s[t]) {
+          ++nl;
+          const int R = oroot_s[t];
+          const bool easy = R >= 0 && tri_in_range(r_s[t]) && tri_need(dl_s[t], oe_s[t]) <= 2.0f;
+          nh += easy ? 0 : 1;
+        }
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        nh += __shfl_xor_sync(0xffffffffu, nh, o);
+        nl += __shfl_xor_sync(0xffffffffu, nl, o);
+      }
+      int *red = reinterpret_cast<int *>(wtop);   // idle between updates
+      if (lane == 0) {
+        red[2 * warp] = nh;
+        red[2 * warp + 1] = nl;
+      }
+      __syncthreads();
+      if (warp == 0) {
+        int h = 0, l = 0;
+#pragma unroll
+        for (int w8 = 0; w8 < kSelectWarps; ++w8) {
+          h += red[2 * w8];
+          l += red[2 * w8 + 1];
+        }
+        if (lane < C) st_cluster_v2f(map_shared(&hard_s[rank], lane), make_float2(__int_as_float(h), __int_as_float(l)));
+      }
+    };
+
     // ---- seed (Eq. 9): one round that accepts argmax w~ ----
     if constexpr (TC) deep_rebuild(false);
     publish(0);
@@ -1349,6 +1415,7 @@ select_kernel(const __grid_constant__ SelectArgs a) {
       if (tri) tri_merge(1, 0);   // the seed is the first root
       update(1, false);
       __syncthreads();
+      if (tri) tri_count();
     }
 
     // ---- rounds (Eq. 10-11) ----
@@ -1356,7 +1423,19 @@ select_kernel(const __grid_constant__ SelectArgs a) {
       const int par = round & 1;
       publish(par);
       cluster_sync();
+      // the root table this round only if most live tokens of the request are not hard
+      // (the counts were sent before the barrier above; every CTA decides alike)
+      bool table_on = false;
       if (tri) {
+        int hs = 0, ls = 0;
+        for (int q = 0; q < C; ++q) {
+          hs += hard_s[q].x;
+          ls += hard_s[q].y;
+        }
+        table_on = 2 * hs <= ls;
+      }
+      tr_s0 = tr_cnt = tr_nts = tr_pre = 0;
+      if (table_on) {
         // this round's slice of the roots: its rows start streaming now, while the
         // candidate list is built (every ring stage is free at a round's start).  The
         // barrier above orders the last merge's root-row copies (any CTA) before these
@@ -1429,18 +1508,22 @@ select_kernel(const __grid_constant__ SelectArgs a) {
       const int nL = (int)misc[1];
       if (!early) stage_list(nL);
       wait_rows();
+      if constexpr (TC) fence_proxy_async_smem();   // the list rows are MMA operands next
       __syncthreads();
       // pairwise dots of L, split over the cluster (4 interleaved pairs per warp),
-      // broadcast to every CTA.  With the tensor-core update the list's Gram is first
-      // taken on the tensor cores: a pair whose tensor-core distance is at least
-      // tc_eps above both members' delta can lower neither member's delta during the
-      // replay (delta only shrinks), so its dot is stored as -inf (distance +inf) and
-      // only the other pairs are evaluated in the canonical order.
+      // broadcast to every CTA.  With the tensor-core update and more pairs than the
+      // cluster's warps take in one pass, the list's Gram is first taken on the
+      // tensor cores: a pair whose tensor-core distance is at least tc_eps above both
+      // members' delta can lower neither member's delta during the replay (delta only
+      // shrinks), so its dot is stored as -inf (distance +inf) and only the other
+      // pairs are evaluated in the canonical order.  When one pass covers every pair
+      // the Gram would only add its latency.
       {
         const int npairs = nL * (nL - 1) / 2;
         int nwork = npairs;              // pairs evaluated exactly
         int *plist = reinterpret_cast<int *>(smem + S.plist);
-        if constexpr (TC) {
+        const bool use_gram = TC && npairs > C * kSelectWarps * 4;
+        if constexpr (TC) if (use_gram) {
           float *gram = reinterpret_cast<float *>(smem + S.gram);
           fence_proxy_async_smem();
           tc_fence_before();
@@ -1516,13 +1599,30 @@ select_kernel(const __grid_constant__ SelectArgs a) {
           }
           nwork = base;
         }
-        for (int p0 = ((int)rank + C * warp) * 4; p0 < nwork; p0 += C * kSelectWarps * 4) {
+        // From here on threads 32 and 64 feed the root table until it is complete (its
+        // copies and MMAs overlap the pair dots and the replay); warps 1 and 2 then
+        // take no pairs, and the two service threads arrive at the cluster barrier
+        // before their work (they write no pair dots) and wait on it after.
+        // The split of the pairs over the warps must be the same in every CTA, so it
+        // depends on the request's root count (the same everywhere), not on whether
+        // this CTA's slice of the roots is empty.
+        const bool tsvc = table_on && nroot > 0;
+        const bool svc = tsvc && tr_nts > 0 && (threadIdx.x == 32 || threadIdx.x == 64);
+        const int nwk = tsvc ? kSelectWarps - 2 : kSelectWarps;   // pair workers per CTA
+        const int wk = (tsvc && warp > 0) ? warp - 2 : warp;       // this warp's worker index
+        if (svc) {
+          cluster_arrive_release();
+          if (threadIdx.x == 32) table_mma(true);
+          else table_load(tr_nts, true);
+        }
+        if (!(tsvc && (warp == 1 || warp == 2)))
+        for (int p0 = ((int)rank + C * wk) * 4; p0 < nwork; p0 += C * nwk * 4) {
           int ja[4], jv[4];   // cbuf rows of the two members of each pair
           int pj[4];          // pair index of each work item
 #pragma unroll
           for (int j = 0; j < 4; ++j) {
             const int wi = min(p0 + j, nwork - 1);
-            const int p = TC ? plist[wi] : wi;
+            const int p = use_gram ? plist[wi] : wi;
             pj[j] = p;
             int u = 0, rem = p;
             while (rem >= nL - 1 - u) { rem -= nL - 1 - u; ++u; }
@@ -1562,13 +1662,13 @@ select_kernel(const __grid_constant__ SelectArgs a) {
               st_cluster_f32(map_shared(&pairbuf[par * kMaxPairs + pj[j]], lane), d);
           }
         }
+        // the pair dots are visible cluster-wide after this barrier (non-aligned: the
+        // service threads arrived early)
+        if (!svc) cluster_arrive_release();
+        cluster_wait_acquire();
       }
-      table_poll();
-      cluster_sync();
       // replay the greedy on L (warp 0; lane u holds member u); meanwhile the root
       // table's service threads finish its copies and MMAs
-      if (tri && tr_nts > 0 && threadIdx.x == 32) table_mma(true);
-      else if (tri && tr_nts > 0 && threadIdx.x == 64) table_load(tr_nts, true);
       if (warp == 0) {
         const unsigned long long Up = misc[0];
         bool pending = lane < nL;
@@ -1612,7 +1712,7 @@ select_kernel(const __grid_constant__ SelectArgs a) {
       __syncthreads();
       if (taken < K) {
         const int nroot_start = nroot;
-        if (tri) {
+        if (table_on) {
           if (warp == 0) {   // cbuf row -> accepted slot
             if (lane < kLcap) rowj_s[lane] = -1;
             __syncwarp();
@@ -1629,10 +1729,13 @@ select_kernel(const __grid_constant__ SelectArgs a) {
           tc_fence_before();
           cluster_sync();
           tc_fence_after();
-          tri_merge(nA, nroot_start);
         }
-        update(nA, tri && nroot_start > 0);
+        // without a table this round no root is known near the new centres: each
+        // becomes a root (while the request has room)
+        if (tri) tri_merge(nA, table_on ? nroot_start : 0);
+        update(nA, table_on && nroot_start > 0);
         __syncthreads();
+        if (tri) tri_count();
       } else if (tri && tr_nts > 0) {
         // the selection ended this round: the table's copies and MMAs still complete
         // (nothing may be in flight when the CTA exits)

@@ -131,6 +131,10 @@ bool encode_x_map(CUtensorMap *m, const void *x, long long rows, int dv, int box
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Bytes of feature rows a CTA streams in one dense update below which the
+// selection does not skip rows by the triangle inequality.
+constexpr double kTriMinStreamBytes = 2.0 * 1024 * 1024;
+
 // Opt-in shared memory per CTA of the sm_100 class, for checks made before a
 // device is at hand.
 constexpr int kSmemOptinSm100 = 232448;
@@ -212,11 +216,13 @@ cudaError_t launch_select(const Plan &pl, const float *w, const void *x, int32_t
       const int tiles = (tpc_c + kTcBM - 1) / kTcBM;
       // stages of kps boxes: the largest kps (<= 4) that still leaves 2 stages
       for (int lc = (c <= 4 ? kLcap : kLcap / 2); lc >= kLcap / 2 && lcap_c == 0; lc /= 2) {
-        // Row skipping: a CTA's slice of the roots takes TMEM columns of the tile
-        // accumulators (at most 128, whole groups of 16), so the request's roots are
-        // capped at that slice times the cluster size.
-        const int s_cap = std::min(128, tiles * lc / kRootGroup * kRootGroup);
-        const int roots_lc = (pl.root_rows > 0 && s_cap >= kRootGroup) ? std::min(kMaxRoots, s_cap * c) : 0;
+        // Row skipping: a CTA's slice of the roots is the M = 128 operand of its
+        // root-table MMA, so the request's roots are capped at 128 per CTA.  It is
+        // used only where a CTA's dense update streams at least kTriMinStreamBytes:
+        // below that the per-round root table costs about what it saves (measured on
+        // 576-token requests in clusters of two).
+        const bool tri_c = pl.root_rows > 0 && (double)tpc_c * rb >= kTriMinStreamBytes;
+        const int roots_lc = tri_c ? std::min(kMaxRoots, kTcBM * c) : 0;
         const size_t fixed = select_smem(0, rb, tpc_c, 0, tb_c, pl.elem, lc, 1, 0, 1, roots_lc).total;
         // TMEM: lc columns per tile plus kGramChains x lc for the list's Gram
         if (fixed + 2 * (size_t)kTcBoxBytes > (size_t)di.optin ||
