@@ -62,10 +62,13 @@
  *             q-heads of 128); num_layers * num_q_heads <= 6144.
  *   selection feat_dim a multiple of 8, at most 2048; the greedy selection
  *             (last_select, last_prune) keeps per-token state of a request in
- *             the shared memory of up to 16 clustered CTAs, which bounds N_b:
- *             about 128K tokens at feat_dim 64, 72K at bf16 feat_dim 2048,
- *             13K at fp32 feat_dim 2048.  Top-k and the gather have no such
- *             bound.
+ *             the shared memory of up to 16 clustered CTAs: about 120K tokens
+ *             at feat_dim 64, 72K at bf16 feat_dim 2048, 13K at fp32 feat_dim
+ *             2048.  A call of at most 4 requests past that bound runs them on
+ *             every SM of the GPU instead (per-token state spread over all
+ *             CTAs: millions of tokens); a call of more requests returns
+ *             LAST_ERR_UNSUPPORTED for them.  Top-k and the gather have no
+ *             such bound.
  */
 #ifndef LAST_H_
 #define LAST_H_

@@ -118,6 +118,8 @@ last_status make_plan(const last_problem *p, bool need_scores, bool need_select,
   o = align_up(o + sizeof(int32_t) * 2 * std::max(pl->total_chunks, 1));
   pl->off_order = o;
   o = align_up(o + sizeof(int32_t) * std::max(B, 1));
+  pl->off_gbar = o;   // abort word and one barrier counter per request slot
+  o = align_up(o + sizeof(uint32_t) * (1 + kGridMaxReq));
   const size_t blob_end = o;
   pl->off_stats = o;
   o = align_up(o + sizeof(float) * 4 * (size_t)std::max(pl->L, 0) * std::max(pl->Hq, 0) *
@@ -143,6 +145,9 @@ last_status make_plan(const last_problem *p, bool need_scores, bool need_select,
   o = align_up(o + (size_t)pl->root_rows * (size_t)((std::max(p->feat_dim, 0) + 63) / 64) * 128);
   pl->off_rtab = o;
   o = align_up(o + (size_t)pl->root_rows * kRootTableCols * sizeof(float));
+  // the whole-GPU selection's published keys, for launches that may take it
+  pl->off_gpub = o;
+  if (B <= kGridMaxReq && pl->max_vis >= kGridMinTokens) o = align_up(o + grid_pub_bytes());
   pl->total_bytes = o;
 
   // ---- host staging: [err words][meta][items][order], one copy ----

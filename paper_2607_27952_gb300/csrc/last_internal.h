@@ -32,6 +32,8 @@ constexpr int kMaxFeatDim = 2048;    // selection keeps x_j in 64 fp32 registers
 constexpr int kRootsPerRequest = 1024;   // root rows per request (the selection's kMaxRoots)
 constexpr int kRootTableCols = 32;       // bound-table columns per root (the selection's kMaxAccept)
 constexpr int kSelectWarps = 8;
+constexpr int kGridMaxReq = 4;      // requests of one whole-GPU selection launch
+constexpr int kGridMaxCtas = 256;   // CTAs of one whole-GPU selection launch at most
 constexpr int kGatherThreads = 256;
 
 // Device error flags (first word of the workspace).
@@ -54,6 +56,9 @@ struct Plan {
   // bf16 selection scratch: root rows [root_rows][dv] and the bound table
   // [root_rows][kRootTableCols] (after the scoring scratch; score_bytes excludes them)
   size_t off_roots = 0, off_rtab = 0, score_bytes = 0;
+  // whole-GPU selection: barrier counters (zeroed with the staged plan) and the
+  // published keys
+  size_t off_gbar = 0, off_gpub = 0;
   long long root_rows = 0;
   // host staging (error word, meta rows, score items, selection order) in ws order
   std::vector<int32_t> host_blob;
@@ -77,6 +82,18 @@ cudaError_t launch_select(const Plan &pl, const float *w, const void *x, int32_t
                           void *x_out, char *ws, cudaStream_t s);
 cudaError_t launch_gather(const Plan &pl, const void *x, const int32_t *idx, void *x_out,
                           char *ws, cudaStream_t s);
+// The whole-GPU selection of a few long requests (select_grid.cu).
+cudaError_t launch_select_grid(const Plan &pl, const float *w, const void *x, int32_t *idx_out,
+                               void *x_out, char *ws, cudaStream_t s);
+size_t grid_select_smem(int row_bytes, int tpc);
+size_t grid_pub_bytes();
+// Whether the whole-GPU selection can run the plan's requests on the current device
+// (it takes requests too long for any thread-block cluster, at most kGridMaxReq).
+bool grid_select_fits(const Plan &pl);
+// Requests shorter than this always fit a cluster: their workspace needs no
+// room for the whole-GPU selection.
+constexpr int kGridMinTokens = 4096;
+
 cudaError_t launch_topk(const Plan &pl, const float *w, int32_t *idx_out, char *ws,
                         cudaStream_t s);
 

@@ -156,10 +156,13 @@ bool select_supported(const Plan &pl, std::string *why) {
 bool select_fits(const Plan &pl, std::string *why) {
   // The largest request: the CUDA-core update's per-token state of one of 16
   // clustered CTAs, with a row ring and no row cache, within sm_100-class shared
-  // memory (the launch itself takes the device's own figure).
+  // memory (the launch itself takes the device's own figure).  Past that, up to
+  // kGridMaxReq requests run on the whole GPU (select_grid.cu) when their tokens
+  // fit its CTAs' shared memory.
   const int tpc = (pl.max_vis + kMaxCluster - 1) / kMaxCluster;
   const int tb = select_tb(pl.elem, false, tpc);
-  if (select_smem(0, pl.dv * pl.elem, tpc, 1, tb, pl.elem, kLcap / 2).total > (size_t)kSmemOptinSm100) {
+  if (select_smem(0, pl.dv * pl.elem, tpc, 1, tb, pl.elem, kLcap / 2).total > (size_t)kSmemOptinSm100 &&
+      !(pl.B <= kGridMaxReq && grid_select_fits(pl))) {
     if (why) *why = "a request has too many visual tokens for the selection's shared-memory plan";
     return false;
   }
@@ -282,7 +285,12 @@ cudaError_t launch_select(const Plan &pl, const float *w, const void *x, int32_t
     }
   }
   }
-  if (C == 0) return cudaErrorInvalidConfiguration;
+  if (C == 0) {
+    // requests too long for any cluster: up to kGridMaxReq of them on the whole GPU
+    if (pl.B <= kGridMaxReq && grid_select_fits(pl))
+      return launch_select_grid(pl, w, x, idx_out, x_out, ws, s);
+    return cudaErrorInvalidConfiguration;
+  }
   cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   if (e != cudaSuccess) return e;
   e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);

@@ -73,10 +73,14 @@ def test_scores_rejects_bad_problems_before_launch(lib, kw, status):
     (dict(feat_dim=100), last.LAST_ERR_INVALID_ARG),
     (dict(feat_dim=4096), last.LAST_ERR_UNSUPPORTED),
     (dict(cu_vis=[0, 6, 5]), last.LAST_ERR_INVALID_ARG),
-    (dict(dtype="f32", feat_dim=2048, cu_seqlens=[0, 10, 20020], cu_vis=[0, 6, 20006]),
-     last.LAST_ERR_UNSUPPORTED),                                             # N_b past smem
-    (dict(feat_dim=64, cu_seqlens=[0, 10, 140020], cu_vis=[0, 6, 140006]),
-     last.LAST_ERR_UNSUPPORTED),
+    # N_b past the clustered plan's shared memory, in a launch of five requests (the
+    # whole-GPU selection takes at most four)
+    (dict(dtype="f32", feat_dim=2048, batch=5, cu_seqlens=[0, 10, 20020, 20030, 20040, 20050],
+          vis_start=[0, 2, 0, 0, 0], cu_vis=[0, 6, 20006, 20007, 20008, 20009],
+          cu_keep=[0, 2, 5, 6, 7, 8]), last.LAST_ERR_UNSUPPORTED),
+    (dict(feat_dim=64, batch=5, cu_seqlens=[0, 10, 140020, 140030, 140040, 140050],
+          vis_start=[0, 2, 0, 0, 0], cu_vis=[0, 6, 140006, 140007, 140008, 140009],
+          cu_keep=[0, 2, 5, 6, 7, 8]), last.LAST_ERR_UNSUPPORTED),
 ])
 def test_select_rejects_bad_problems_before_launch(lib, kw, status):
     prob = _problem(**kw)
