@@ -42,7 +42,7 @@ constexpr int kGridTop = 17;       // keys each CTA publishes: 16 candidates and
 constexpr int kGridLcap = 16;      // candidate list
 constexpr int kGridPairs = kGridLcap * (kGridLcap - 1) / 2;
 constexpr int kGridAccept = 16;    // picks accepted per round at most
-constexpr uint32_t kGridWaitLimit = 1u << 21;   // polls of one barrier wait (about a second)
+constexpr uint32_t kGridWaitLimit = 1u << 21;   // polls of one barrier wait (a second or two)
 
 struct GridArgs {
   const void *x;
@@ -137,7 +137,6 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_grid_kernel(const __gri
       for (uint32_t i = 0; i < kGridWaitLimit; ++i) {
         if (ld_acquire_u32(ctr) >= target) { ok = true; break; }
         if (ld_acquire_u32(abort_w) != 0u) break;
-        __nanosleep(32);
       }
       if (!ok) {
         atomicOr(a.err, kErrTimeout);
@@ -265,19 +264,23 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_grid_kernel(const __gri
           misc[0] = cut > U ? cut : U;   // U' bounds every token outside the list
           misc[1] = (unsigned long long)n;
         }
-        // the members' (delta, w~, 1/|x|) from their owners' published payload
-        if (lane < n) {
-          const unsigned long long key = lp_key[lane];
-          const int gi = key_index(key);
-          const int owner = min(G - 1, gi / tpc);
-          const size_t ob = ((size_t)par * kGridMaxCtas + a.cta0[slot] + owner) * kGridTop;
-          float4 f = make_float4(0.f, 0.f, 0.f, 0.f);
-          for (int e = 0; e < kGridTop - 1; ++e)
-            if (__ldcg(a.pub_key + ob + e) == key) f = __ldcg(a.pub_f + ob + e);
-          lp_idx[lane] = gi;
-          lp_f[lane * 3 + 0] = f.x;
-          lp_f[lane * 3 + 1] = f.y;
-          lp_f[lane * 3 + 2] = f.z;
+        if (lane < n) lp_idx[lane] = key_index(lp_key[lane]);
+      }
+      __syncthreads();
+      // the members' (delta, w~, 1/|x|) from the published payload: every thread
+      // matches its share of the request's published entries against the list
+      {
+        const int n = (int)misc[1];
+        for (int f = threadIdx.x; f < G * kGridTop; f += kSelThreads) {
+          if (f % kGridTop == kGridTop - 1) continue;
+          const unsigned long long v = __ldcg(a.pub_key + base + f);
+          for (int u = 0; u < n; ++u)
+            if (v == lp_key[u]) {
+              const float4 pf = __ldcg(a.pub_f + base + f);
+              lp_f[u * 3 + 0] = pf.x;
+              lp_f[u * 3 + 1] = pf.y;
+              lp_f[u * 3 + 2] = pf.z;
+            }
         }
       }
       __syncthreads();
@@ -372,48 +375,85 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_grid_kernel(const __gri
       continue;
     }
     // delta <- min(delta, d(i, c)) over the accepted centres in acceptance order,
-    // four centres at a time (independent canonical fma chains) per warp and token
-    for (int t = warp; t < nloc; t += kSelectWarps) {
-      if (sel_s[t]) continue;
-      float xv[NCH][8];
-      const char *row = xg + (long long)t * rb;
-#pragma unroll
-      for (int g = 0; g < NCH; ++g) {
-        const int col = 256 * g + 8 * lane;
-        if (col < dv) load8<T, false>(row, col, xv[g]);
-        else
-#pragma unroll
-          for (int e = 0; e < 8; ++e) xv[g][e] = 0.f;
-      }
-      const float ri = r_s[t];
-      float dl = dl_s[t];
-      for (int j0 = 0; j0 < nA; j0 += 4) {
-        float acc[4] = {0.f, 0.f, 0.f, 0.f};
+    // four centres at a time (independent canonical fma chains) per warp and token;
+    // the warp's next token row is in flight while the current one is evaluated
+    {
+      constexpr bool kBf16 = sizeof(T) == 2;
+      constexpr int kVec = kBf16 ? 1 : 2;   // 16-byte vectors per 8-coordinate group
+      auto load_tok = [&](int t, U4 (*xv)[kVec]) {
+        const char *row = xg + (long long)t * rb;
 #pragma unroll
         for (int g = 0; g < NCH; ++g) {
           const int col = 256 * g + 8 * lane;
-          if (col < dv) {
 #pragma unroll
-            for (int j = 0; j < 4; ++j) {
-              if (j0 + j < nA) {
-                float ec[8];
-                load8<T, true>(cbuf + (long long)acc_s[j0 + j] * rb, col, ec);
+          for (int h = 0; h < kVec; ++h)
+            xv[g][h] = col < dv ? ldg_stream(row + col * (int)sizeof(T) + 16 * h) : U4{0, 0, 0, 0};
+        }
+      };
+      auto eval_tok = [&](int t, U4 (*xv)[kVec]) {
+        const float ri = r_s[t];
+        float dl = dl_s[t];
+        for (int j0 = 0; j0 < nA; j0 += 4) {
+          float acc[4] = {0.f, 0.f, 0.f, 0.f};
+          const char *crow[4];
 #pragma unroll
-                for (int e = 0; e < 8; ++e) acc[j] = __fmaf_rn(xv[g][e], ec[e], acc[j]);
+          for (int j = 0; j < 4; ++j) crow[j] = cbuf + (long long)acc_s[min(j0 + j, nA - 1)] * rb;
+#pragma unroll
+          for (int g = 0; g < NCH; ++g) {
+            const int col = 256 * g + 8 * lane;
+            if (col < dv) {
+#pragma unroll
+              for (int j = 0; j < 4; ++j) {
+                if (kBf16) {
+                  const U4 cv = lds(crow[j] + col * 2);
+                  const uint32_t xw[4] = {xv[g][0].x, xv[g][0].y, xv[g][0].z, xv[g][0].w};
+                  const uint32_t cw[4] = {cv.x, cv.y, cv.z, cv.w};
+#pragma unroll
+                  for (int hw = 0; hw < 4; ++hw) {
+                    acc[j] = fma_bf16_lo(xw[hw], cw[hw], acc[j]);
+                    acc[j] = fma_bf16_hi(xw[hw], cw[hw], acc[j]);
+                  }
+                } else {
+                  float ec[8], ex[8];
+                  load8<T, true>(crow[j], col, ec);
+                  Elem<T>::widen(xv[g][0], ex);
+                  Elem<T>::widen(xv[g][kVec - 1], ex + 4);
+#pragma unroll
+                  for (int e = 0; e < 8; ++e) acc[j] = __fmaf_rn(ex[e], ec[e], acc[j]);
+                }
               }
             }
           }
-        }
 #pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          if (j0 + j < nA) {
-            const float dot = butterfly_sum(acc[j]);
-            const float rc = lp_f[acc_s[j0 + j] * 3 + 2];
-            dl = fminf(dl, __fsub_rn(1.0f, __fmul_rn(__fmul_rn(dot, ri), rc)));
+          for (int j = 0; j < 4; ++j) {
+            if (j0 + j < nA) {
+              const float dot = butterfly_sum(acc[j]);
+              const float rc = lp_f[acc_s[j0 + j] * 3 + 2];
+              dl = fminf(dl, __fsub_rn(1.0f, __fmul_rn(__fmul_rn(dot, ri), rc)));
+            }
           }
         }
+        if (lane == 0) dl_s[t] = dl;
+      };
+      // the warp's live tokens t = warp, warp + 8, ... (selected ones skipped)
+      auto next_live = [&](int t) {
+        while (t < nloc && sel_s[t]) t += kSelectWarps;
+        return t;
+      };
+      U4 xa[NCH][kVec], xb[NCH][kVec];
+      int t = next_live(warp);
+      if (t < nloc) load_tok(t, xa);
+      while (t < nloc) {
+        int tn = next_live(t + kSelectWarps);
+        if (tn < nloc) load_tok(tn, xb);
+        eval_tok(t, xa);
+        t = tn;
+        if (t >= nloc) break;
+        tn = next_live(t + kSelectWarps);
+        if (tn < nloc) load_tok(tn, xa);
+        eval_tok(t, xb);
+        t = tn;
       }
-      if (lane == 0) dl_s[t] = dl;
     }
     __syncthreads();
   }
