@@ -31,6 +31,10 @@
  *   - Calls are asynchronous on `stream` (a cudaStream_t; NULL = legacy
  *     default stream).  Successive calls on one stream may reuse one
  *     workspace; concurrent calls need distinct workspaces.
+ *   - No entry point may be captured into a CUDA graph: each call copies its
+ *     plan from pageable host memory that it owns and releases on return, so
+ *     a captured copy would replay freed memory.  Launch-bound callers batch
+ *     requests into one call instead (one launch per kernel for the batch).
  *   - Argument errors are detected on the host before any launch; the call
  *     returns a status and touches no output.  Device-side checks set a flag in
  *     the workspace that last_poll() reports: an out-of-range caller index
@@ -201,9 +205,10 @@ last_status last_prune_host(const last_problem *p, const void *q_host, const voi
  * treats later allocations as failures, or a program without a device allocator
  * of its own.  Same inputs, outputs and results as last_scores; the scratch lives
  * in a fixed 16 MiB array inside the library, held on every GPU that loads the
- * library until the process exits.  The first call on each device looks up that
- * array's device address (cudaGetSymbolAddress) with the device current; make
- * that first call before any stream capture on that device.  All calls share
+ * library until the process exits.  Each call looks up that array's device
+ * address (cudaGetSymbolAddress, cached per device after the first call) with
+ * the device current; like every entry point it cannot be captured into a CUDA
+ * graph (the plan is copied from host memory the call releases).  All calls share
  * the array and it keeps the last call's contents: calls whose executions
  * overlap on the GPU race on it.  A problem needing more than 16 MiB of scratch
  * (last_workspace_size) returns LAST_ERR_UNSUPPORTED.  Allocates nothing. */
