@@ -144,7 +144,7 @@ def workload_desc(wl, budget, name="c5"):
 
 
 def prune_bytes_moved(wl):
-    """Bytes under SURVEY-style "bytes moved" accounting of the fused prune:
+    """Bytes of the fused prune under a "bytes moved" accounting:
     compulsory bytes (K, q and X read once, w~ written, X_S written and its rows
     read) plus the greedy's notional feature reads, k_b * N_b * d_v elements per
     request (the O(K N d_v) distance work of Sec. 3.4).  The notional reads never
@@ -704,7 +704,7 @@ def main():
                               "note": "compulsory_frac = the step's unavoidable HBM bytes (K, q, "
                                       "X once, w~, kept rows) over the step time, of measured "
                                       "HBM; greedy_effective_TBps values the greedy's notional "
-                                      "k N d_v feature reads at HBM rate (SURVEY accounting) "
+                                      "k N d_v feature reads at HBM rate (bytes-moved accounting) "
                                       "and is not a fraction of any roof: most of those pairs "
                                       "are skipped or served on chip"},
         "paper_context": PAPER_CONTEXT,
