@@ -123,6 +123,7 @@ struct SelectArgs {
   char *roots;           // root row groups: request b's from row meta kRootOff (a multiple of 16)
   float *rtab;           // per round: rho lower bounds [root row][kMaxAccept]
   int tri;               // 1: skip rows by the triangle inequality
+  int gram;              // tc: 1 when the list's Gram may be taken (its buffers exist)
   int root_cap;          // roots per request (<= kMaxRoots, <= s_cap * csize)
   float tri_eps_x;       // bound on |root-table distance - exact distance| (tc_eps + kTriEpsC)
 };
@@ -147,7 +148,8 @@ __host__ __device__ inline int blocks_per_warp(int tpc_max, int tb) {
 __host__ __device__ inline SelectSmem select_smem(int cache_rows, int row_bytes, int tpc_max,
                                                   int ring, int tb, int elem, int lcap,
                                                   int tc = 0, int stages = 0, int kps = 1,
-                                                  int roots = 0) {
+                                                  int roots = 0, int csize = kMaxCluster,
+                                                  int gram = 1) {
   SelectSmem s;
   size_t o = 0;
   if (tc) {
@@ -169,11 +171,11 @@ __host__ __device__ inline SelectSmem select_smem(int cache_rows, int row_bytes,
   s.w = o; o += align16(sizeof(float) * tpc_max);
   s.r = o; o += align16(sizeof(float) * tpc_max);
   s.dl = o; o += align16(sizeof(float) * tpc_max);
-  s.list = o; o += align16(sizeof(int) * tpc_max);
+  s.list = o; o += tc ? 0 : align16(sizeof(int) * tpc_max);   // tensor-core variant: aliases fidx
   s.sel = o; o += align16(tpc_max);
   s.wtop = o; o += sizeof(unsigned long long) * kSelectWarps * kTopMax;
-  s.pub_key = o; o += sizeof(unsigned long long) * 2 * kMaxCluster * kTopMax;
-  s.pub_f = o; o += sizeof(float4) * 2 * kMaxCluster * kTopMax;
+  s.pub_key = o; o += sizeof(unsigned long long) * 2 * csize * kTopMax;   // [parity][CTA][entry]
+  s.pub_f = o; o += sizeof(float4) * 2 * csize * kTopMax;
   s.lp_key = o; o += sizeof(unsigned long long) * kLcap;
   s.lp_f = o; o += sizeof(float) * kLcap * 3;
   s.lp_idx = o; o += sizeof(int) * kLcap;
@@ -188,16 +190,18 @@ __host__ __device__ inline SelectSmem select_smem(int cache_rows, int row_bytes,
   o = align16(o);   // later regions take 16-byte vector accesses (mr: v4 loads and cluster stores)
   s.tslot = o; o += tc ? 16 : 0;
   s.fidx = o; o += tc ? align16(sizeof(int) * tpc_max) : 0;
+  if (tc) s.list = s.fidx;   // the epilogue's list of kept tokens, after the last update
   s.fmask = o; o += tc ? align16(sizeof(uint32_t) * tpc_max) : 0;
   s.fcnt = o; o += tc ? 16 : 0;
-  s.gram = o; o += tc ? sizeof(float) * kLcap * kLcap : 0;       // list Gram (tensor cores)
-  s.plist = o; o += tc ? align16(sizeof(int) * (kMaxPairs + 1)) : 0;   // pairs to evaluate
+  // list Gram (tensor cores) and the pairs it leaves, when the launch may take it
+  s.gram = o; o += tc && gram ? sizeof(float) * kLcap * kLcap : 0;
+  s.plist = o; o += tc && gram ? align16(sizeof(int) * (kMaxPairs + 1)) : 0;
   // triangle-inequality state: per token the root of its nearest centre and the bound
   // e of that centre; per root the round's smallest rho lower bound and its 1/|x|;
   // per accepted centre its root and e; the cluster's partial nearest-root searches
   // (sized 0 when the launch does not skip rows: roots == 0)
   const bool tri = tc && roots > 0;
-  s.oroot = o; o += tri ? align16(sizeof(int) * tpc_max) : 0;
+  s.oroot = o; o += tri ? align16(sizeof(int16_t) * tpc_max) : 0;   // roots < 2^15
   s.oe = o; o += tri ? align16(sizeof(float) * tpc_max) : 0;
   s.mr = o; o += tri ? align16(sizeof(float) * roots) : 0;
   s.rootr = o; o += tri ? align16(sizeof(float) * roots) : 0;
@@ -337,7 +341,7 @@ select_kernel(const __grid_constant__ SelectArgs a) {
 
   const SelectSmem S = select_smem(a.cache_rows, a.row_bytes, a.tpc_max, a.ring, TB, (int)sizeof(T),
                                    a.lcap, TC ? 1 : 0, TC ? a.tc_stages : 0, TC ? a.tc_kps : 1,
-                                   TC && a.tri ? a.root_cap : 0);
+                                   TC && a.tri ? a.root_cap : 0, a.csize, TC ? a.gram : 1);
   {
     // The host sizes the launch with the same plan; should they ever disagree, every
     // CTA of every cluster leaves here together (before any cluster barrier)
@@ -373,7 +377,7 @@ select_kernel(const __grid_constant__ SelectArgs a) {
   int *cnt_s = reinterpret_cast<int *>(smem + S.cnt);
   // triangle-inequality state (tensor-core variant)
   const bool tri = TC && a.tri != 0;
-  int *oroot_s = reinterpret_cast<int *>(smem + S.oroot);
+  int16_t *oroot_s = reinterpret_cast<int16_t *>(smem + S.oroot);
   float *oe_s = reinterpret_cast<float *>(smem + S.oe);
   float *mr_s = reinterpret_cast<float *>(smem + S.mr);
   float *rootr_s = reinterpret_cast<float *>(smem + S.rootr);
@@ -601,7 +605,7 @@ select_kernel(const __grid_constant__ SelectArgs a) {
         if (lane < C) {
           for (int i = 0; i <= a.mc; ++i) {
             const unsigned long long key = top5[i];
-            const int slot = (par * kMaxCluster + (int)rank) * kTopMax + i;
+            const int slot = (par * C + (int)rank) * kTopMax + i;
             float4 f = make_float4(0.f, 0.f, 0.f, 0.f);
             if (key != 0ull) {
               const int lt = key_index(key) - lo;
@@ -1059,7 +1063,7 @@ select_kernel(const __grid_constant__ SelectArgs a) {
         if (lane == 0) {
           dl_s[t] = dl;
           if (tri && own >= 0) {
-            oroot_s[t] = croot_s[own];
+            oroot_s[t] = (int16_t)croot_s[own];
             oe_s[t] = ce_s[own];
           }
         }
@@ -1392,10 +1396,10 @@ select_kernel(const __grid_constant__ SelectArgs a) {
       unsigned long long best = 0ull;
       int bq = 0;
       for (int q = 0; q < C; ++q) {
-        const unsigned long long kq = pub_key[(0 * kMaxCluster + q) * kTopMax];
+        const unsigned long long kq = pub_key[q * kTopMax];
         if (kq > best) { best = kq; bq = q; }
       }
-      const int slot = (0 * kMaxCluster + bq) * kTopMax;
+      const int slot = bq * kTopMax;
       lp_key[0] = best;
       lp_idx[0] = key_index(best);
       const float4 f = pub_f[slot];
@@ -1450,7 +1454,7 @@ select_kernel(const __grid_constant__ SelectArgs a) {
       if (TC && early && warp > 0) {   // warps 1.. copy while warp 0 builds the list
         for (int q = 0; q < C; ++q)
           for (int e = 0; e < a.mc; ++e) {
-            const unsigned long long kq = pub_key[(par * kMaxCluster + q) * kTopMax + e];
+            const unsigned long long kq = pub_key[(par * C + q) * kTopMax + e];
             if (kq != 0ull) copy_row_tc(q * a.mc + e, key_index(kq), 32, kSelThreads - 32);
           }
         cp_async_commit();
@@ -1458,11 +1462,11 @@ select_kernel(const __grid_constant__ SelectArgs a) {
         uint32_t bytes = 0;
         for (int q = 0; q < C; ++q)
           for (int e = 0; e < a.mc; ++e)
-            bytes += pub_key[(par * kMaxCluster + q) * kTopMax + e] != 0ull ? (uint32_t)rb : 0u;
+            bytes += pub_key[(par * C + q) * kTopMax + e] != 0ull ? (uint32_t)rb : 0u;
         mbar_expect_tx(bar, bytes);
         for (int q = 0; q < C; ++q)
           for (int e = 0; e < a.mc; ++e) {
-            const unsigned long long kq = pub_key[(par * kMaxCluster + q) * kTopMax + e];
+            const unsigned long long kq = pub_key[(par * C + q) * kTopMax + e];
             if (kq != 0ull)
               bulk_g2s(cbuf + (long long)(q * a.mc + e) * rb, xreq + (long long)key_index(kq) * rb,
                        (uint32_t)rb, bar);
@@ -1473,7 +1477,7 @@ select_kernel(const __grid_constant__ SelectArgs a) {
       // holds the head of CTA q's entries and the warp takes the largest head.
       if (warp == 0) {
         const int kPer = a.mc;
-        const int base = (par * kMaxCluster + lane) * kTopMax;
+        const int base = (par * C + lane) * kTopMax;
         const unsigned long long u5 = lane < C ? pub_key[base + kPer] : 0ull;
         const unsigned long long U = warp_max_u64(u5);
         int ptr = 0, n = 0;
@@ -1522,7 +1526,7 @@ select_kernel(const __grid_constant__ SelectArgs a) {
         const int npairs = nL * (nL - 1) / 2;
         int nwork = npairs;              // pairs evaluated exactly
         int *plist = reinterpret_cast<int *>(smem + S.plist);
-        const bool use_gram = TC && npairs > C * kSelectWarps * 4;
+        const bool use_gram = TC && a.gram != 0 && npairs > C * kSelectWarps * 4;
         if constexpr (TC) if (use_gram) {
           float *gram = reinterpret_cast<float *>(smem + S.gram);
           fence_proxy_async_smem();

@@ -199,6 +199,7 @@ cudaError_t launch_select(const Plan &pl, const float *w, const void *x, int32_t
   // TMEM column per list entry and 128-row tile, so very long requests do not
   // fit), the sizes are costed again for the CUDA-core update.
   int C = 0, tpc = 0, cache_rows = 0, ring = 0, lcap = kLcap / 2, stages = 0, kps = 1, roots = 0;
+  int gram = 0;
   size_t smem = 0;
   double best = 0.0;
   void *fn = nullptr;
@@ -211,14 +212,14 @@ cudaError_t launch_select(const Plan &pl, const float *w, const void *x, int32_t
     const int tpc_c = (pl.max_vis + c - 1) / c;
     const int tb_c = select_tb(pl.elem, tc, tpc_c);
     void *fn_c = pick_select(pl.dtype, nch, tb_c, tc);
-    int cache_c = 0, ring_c = 0, lcap_c = 0, stages_c = 0, kps_c = 1, roots_c = 0;
+    int cache_c = 0, ring_c = 0, lcap_c = 0, stages_c = 0, kps_c = 1, roots_c = 0, gram_c = 0;
     size_t smem_c = 0;
     if (tc) {
       // the list length is the MMA N: lcap accumulator columns per 128-row tile; the
       // TMA ring takes the shared memory left over
       const int tiles = (tpc_c + kTcBM - 1) / kTcBM;
       // stages of kps boxes: the largest kps (<= 4) that still leaves 2 stages
-      for (int lc = (c <= 4 ? kLcap : kLcap / 2); lc >= kLcap / 2 && lcap_c == 0; lc /= 2) {
+      for (int lc = kLcap; lc >= kLcap / 2 && lcap_c == 0; lc /= 2) {
         // Row skipping: a CTA's slice of the roots is the M = 128 operand of its
         // root-table MMA, so the request's roots are capped at 128 per CTA.  It is
         // used only where a CTA's dense update streams at least kTriMinStreamBytes:
@@ -226,7 +227,11 @@ cudaError_t launch_select(const Plan &pl, const float *w, const void *x, int32_t
         // 576-token requests in clusters of two).
         const bool tri_c = pl.root_rows > 0 && (double)tpc_c * rb >= kTriMinStreamBytes;
         const int roots_lc = tri_c ? std::min(kMaxRoots, kTcBM * c) : 0;
-        const size_t fixed = select_smem(0, rb, tpc_c, 0, tb_c, pl.elem, lc, 1, 0, 1, roots_lc).total;
+        // the list's Gram only when the pair dots would take more than two passes of
+        // the cluster's pair workers (at least six warps per CTA)
+        const int gram_lc = lc * (lc - 1) / 2 > 2 * c * (kSelectWarps - 2) * 4 ? 1 : 0;
+        const size_t fixed = select_smem(0, rb, tpc_c, 0, tb_c, pl.elem, lc, 1, 0, 1, roots_lc, c,
+                                         gram_lc).total;
         // TMEM: lc columns per tile plus kGramChains x lc for the list's Gram
         if (fixed + 2 * (size_t)kTcBoxBytes > (size_t)di.optin ||
             (tiles + kGramChains) * lc > kTmemCols)
@@ -238,22 +243,24 @@ cudaError_t launch_select(const Plan &pl, const float *w, const void *x, int32_t
         stages_c = (int)std::min<size_t>(kTcMaxStages, room / ((size_t)kps_c * kTcBoxBytes));
         lcap_c = lc;
         roots_c = roots_lc;
-        smem_c = select_smem(0, rb, tpc_c, 0, tb_c, pl.elem, lc, 1, stages_c, kps_c, roots_c).total;
+        gram_c = gram_lc;
+        smem_c = select_smem(0, rb, tpc_c, 0, tb_c, pl.elem, lc, 1, stages_c, kps_c, roots_c, c,
+                             gram_c).total;
       }
       if (lcap_c == 0) continue;
     } else {
       lcap_c = c <= 4 ? kLcap : kLcap / 2;
       // rows that fit without a ring; otherwise reserve the ring and cache what is left
-      const size_t fixed0 = select_smem(0, rb, tpc_c, 0, tb_c, pl.elem, lcap_c).total;
+      const size_t fixed0 = select_smem(0, rb, tpc_c, 0, tb_c, pl.elem, lcap_c, 0, 0, 1, 0, c).total;
       if (fixed0 > (size_t)di.optin) continue;
       cache_c = (int)std::min<size_t>(tpc_c, (di.optin - fixed0) / rb);
       if (cache_c < tpc_c) {
         ring_c = 1;
-        const size_t fixed1 = select_smem(0, rb, tpc_c, 1, tb_c, pl.elem, lcap_c).total;
+        const size_t fixed1 = select_smem(0, rb, tpc_c, 1, tb_c, pl.elem, lcap_c, 0, 0, 1, 0, c).total;
         if (fixed1 > (size_t)di.optin) continue;
         cache_c = (int)std::min<size_t>(tpc_c, (di.optin - fixed1) / rb);
       }
-      smem_c = select_smem(cache_c, rb, tpc_c, ring_c, tb_c, pl.elem, lcap_c).total;
+      smem_c = select_smem(cache_c, rb, tpc_c, ring_c, tb_c, pl.elem, lcap_c, 0, 0, 1, 0, c).total;
     }
     const int active = active_clusters(fn_c, c, smem_c);
     if (active <= 0) continue;
@@ -273,6 +280,10 @@ cudaError_t launch_select(const Plan &pl, const float *w, const void *x, int32_t
       const double share = di.dram_bytes_per_cycle / ctas * (from_hbm ? 1.0 : 2.5);
       const double bw = std::min(std::min(kps_c * (double)kTcBoxBytes / 900.0, 26.0), share);
       round_cycles = bytes / bw + 30000.0 + 400.0 * c;
+      // a 16-entry list accepts fewer consecutive picks per round than a 32-entry
+      // one: a host replay of the rounds on the benchmark presets needs 1.4-1.6x the
+      // rounds (c3, c4 and the video batch), so its rounds are weighted by 1.4
+      if (lcap_c < kLcap) round_cycles *= 1.4;
     } else {
       const double stream_penalty = from_hbm ? 3.0 : 1.0;
       const double streamed = std::max(0, tpc_c - cache_c), cached = std::min(tpc_c, cache_c);
@@ -281,7 +292,7 @@ cudaError_t launch_select(const Plan &pl, const float *w, const void *x, int32_t
     const double cost = waves * round_cycles;
     if (C == 0 || cost < best) {
       best = cost; C = c; tpc = tpc_c; cache_rows = cache_c; smem = smem_c; ring = ring_c;
-      lcap = lcap_c; fn = fn_c; stages = stages_c; kps = kps_c; roots = roots_c;
+      lcap = lcap_c; fn = fn_c; stages = stages_c; kps = kps_c; roots = roots_c; gram = gram_c;
     }
   }
   }
@@ -314,6 +325,7 @@ cudaError_t launch_select(const Plan &pl, const float *w, const void *x, int32_t
   }
   a.ring = ring;
   a.lcap = lcap;
+  a.gram = gram;
   a.err = reinterpret_cast<unsigned *>(ws + pl.off_err);
   if (tc) {
     const int cols = ((tpc + kTcBM - 1) / kTcBM + kGramChains) * lcap;   // tiles + the list Gram
