@@ -218,7 +218,8 @@ cudaError_t launch_select(const Plan &pl, const float *w, const void *x, int32_t
       // the list length is the MMA N: lcap accumulator columns per 128-row tile; the
       // TMA ring takes the shared memory left over
       const int tiles = (tpc_c + kTcBM - 1) / kTcBM;
-      // stages of kps boxes: the largest kps (<= 4) that still leaves 2 stages
+      // stages of kps boxes: the largest kps (<= 4) that still leaves 2 stages.  A list
+      // of kLcap entries is tried first (it accepts more picks per round), then half.
       for (int lc = kLcap; lc >= kLcap / 2 && lcap_c == 0; lc /= 2) {
         // Row skipping: a CTA's slice of the roots is the M = 128 operand of its
         // root-table MMA, so the request's roots are capped at 128 per CTA.  It is
