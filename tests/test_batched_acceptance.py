@@ -1,0 +1,146 @@
+"""The selection kernel's exact batched-acceptance rounds, modelled on the host.
+
+The greedy of Eq. 10-11 takes one pick per step.  The kernel instead runs rounds:
+the request's tokens are split over C CTAs; each CTA publishes its `mc` best keys
+(key = (w_i delta_i, lowest index first on ties)) and its (mc+1)-th key; U is the
+largest of those (mc+1)-th keys, so no unpublished token's key exceeds U; the
+published keys above U form the candidate list L (best first, at most `lcap`),
+and U' = max(U, the first key left out of L) bounds every token outside L for the
+whole round (keys never increase, delta only shrinks).  The round replays the
+greedy on L alone: the member with the largest current key is the true next pick
+while it is above U'; its distances lower the other members' keys; the replay
+stops at U', the budget or the per-round cap.  Then every token's delta takes the
+accepted centres.
+
+This file checks, on a materialised fp64 distance matrix, that the rounds give
+exactly the sequential greedy's picks in order, for cluster sizes 1-12, published
+counts 4-16, lists of 16 and 32 and per-round caps of 16 and 32, on clustered,
+duplicated (exact ties), uniform-weight and video-like features, including k = N.
+It also pins the round counts the design relies on: a longer list never needs
+more rounds on these inputs, and on the video-like request it needs clearly fewer.
+"""
+import numpy as np
+import pytest
+
+NONE = (-np.inf, 0)   # below every key: a CTA with no (mc+1)-th live token
+
+
+def _key(p, i):
+    return (float(p), -int(i))   # larger value first, then the lower index
+
+
+def _sequential(w, dist, k):
+    """Eq. 9-11 step by step: seed argmax w (lowest index on ties), then argmax of
+    w_i min_j d(i, j) over the unselected tokens."""
+    n = len(w)
+    delta = np.full(n, np.inf)
+    sel = np.zeros(n, bool)
+    seq = []
+    for t in range(k):
+        p = w if t == 0 else w * delta
+        best = max((_key(p[i], i) for i in range(n) if not sel[i]))
+        j = -best[1]
+        seq.append(j)
+        sel[j] = True
+        delta = np.minimum(delta, dist[:, j])
+    return seq
+
+
+def _rounds(w, dist, k, C, mc, lcap, max_accept):
+    """The kernel's rounds on the same distances; returns (picks in order, rounds)."""
+    n = len(w)
+    bounds = np.linspace(0, n, C + 1).astype(int)
+    sel = np.zeros(n, bool)
+    seed = -max(_key(w[i], i) for i in range(n))[1]
+    seq = [seed]
+    sel[seed] = True
+    delta = dist[:, seed].copy()
+    rounds = 0
+    while len(seq) < k:
+        rounds += 1
+        p = w * delta
+        pub, U = [], NONE
+        for q in range(C):
+            keys = sorted((_key(p[i], i) for i in range(bounds[q], bounds[q + 1]) if not sel[i]),
+                          reverse=True)
+            pub.extend(keys[:mc])
+            U = max(U, keys[mc] if len(keys) > mc else NONE)
+        above = sorted((kk for kk in pub if kk > U), reverse=True)
+        L = [-kk[1] for kk in above[:lcap]]
+        Up = max(U, above[lcap]) if len(above) > lcap else U
+        cd = {i: delta[i] for i in L}
+        pending = list(L)
+        acc = []
+        while pending and len(seq) + len(acc) < k and len(acc) < max_accept:
+            b = max(pending, key=lambda i: _key(w[i] * cd[i], i))
+            if not _key(w[b] * cd[b], b) > Up:
+                break
+            acc.append(b)
+            pending.remove(b)
+            for i in pending:
+                cd[i] = min(cd[i], dist[i, b])
+        assert acc, "a round must accept the request's best key"
+        for b in acc:
+            sel[b] = True
+            delta = np.minimum(delta, dist[:, b])
+        seq.extend(acc)
+    return seq, rounds
+
+
+def _cos_dist(x):
+    xb = x / np.linalg.norm(x, axis=1, keepdims=True)
+    return 1.0 - xb @ xb.T
+
+
+def _clustered(rng, n, d, nc, noise):
+    c = rng.standard_normal((nc, d))
+    return c[rng.integers(0, nc, n)] + noise * rng.standard_normal((n, d))
+
+
+def _video(rng, frames, per, d, sigma):
+    f = [rng.standard_normal((per, d))]
+    for _ in range(frames - 1):
+        f.append(f[-1] + sigma * rng.standard_normal((per, d)))
+    return np.concatenate(f)
+
+
+def _cases():
+    rng = np.random.default_rng(20260)
+    x = _clustered(rng, 360, 24, 9, 0.15)
+    yield "clustered", x, rng.dirichlet(np.ones(360)), 90
+    base = _clustered(rng, 60, 16, 6, 0.2)
+    x = np.repeat(base, 5, axis=0)                 # every row five times: exact ties
+    yield "duplicates", x, np.repeat(rng.dirichlet(np.ones(60)), 5), 120
+    x = rng.standard_normal((240, 12))
+    yield "uniform-w", x, np.full(240, 1.0 / 240), 240      # k = N
+    x = _video(rng, 8, 48, 32, 0.05)
+    wv = np.repeat(rng.dirichlet(np.ones(48)), 8) * (1 + 0.01 * rng.standard_normal(384))
+    yield "video", x, wv, 200
+
+
+CASES = list(_cases())
+
+
+@pytest.mark.parametrize("name,x,w,k", CASES, ids=[c[0] for c in CASES])
+@pytest.mark.parametrize("C,mc,lcap,max_accept", [
+    (1, 16, 16, 16), (2, 16, 32, 32), (3, 8, 16, 16), (5, 4, 16, 16),
+    (12, 16, 16, 32), (12, 16, 32, 32), (7, 16, 32, 16)])
+def test_rounds_reproduce_the_sequential_greedy(name, x, w, k, C, mc, lcap, max_accept):
+    dist = _cos_dist(x)
+    want = _sequential(w, dist, k)
+    got, rounds = _rounds(w, dist, k, C, mc, lcap, max_accept)
+    assert got == want
+    assert rounds <= k - 1
+
+
+def test_longer_list_needs_fewer_rounds():
+    """The reason for the 32-entry list: with 12 CTAs publishing 16 keys each, a list
+    of 32 accepts more consecutive picks per round than a list of 16 (here on
+    video-like frames, where near-copies of a pick leave the list together)."""
+    for name, x, w, k in CASES:
+        dist = _cos_dist(x)
+        r16 = _rounds(w, dist, k, 12, 16, 16, 32)[1]
+        r32 = _rounds(w, dist, k, 12, 16, 32, 32)[1]
+        assert r32 <= r16, name
+        if name == "video":
+            assert r32 < 0.8 * r16, (r16, r32)
