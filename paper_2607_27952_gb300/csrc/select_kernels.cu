@@ -134,6 +134,8 @@ bool encode_x_map(CUtensorMap *m, const void *x, long long rows, int dv, int box
 // Bytes of feature rows a CTA streams in one dense update below which the
 // selection does not skip rows by the triangle inequality.
 constexpr double kTriMinStreamBytes = 2.0 * 1024 * 1024;
+// the selection keeps each token's nearest root id in 16 bits
+static_assert(kMaxRoots <= 32767, "root ids must fit int16_t");
 
 // Opt-in shared memory per CTA of the sm_100 class, for checks made before a
 // device is at hand.
