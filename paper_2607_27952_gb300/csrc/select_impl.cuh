@@ -575,9 +575,11 @@ select_kernel(const __grid_constant__ SelectArgs a) {
     auto publish = [&](int par) {
       if (warp == 0) {
         if constexpr (TC) {
-          // the candidate list holds the CTA's top keys (at least mc + 1 of them, or
-          // every live token)
-          if (lane < kTop) top5[lane] = lane < d_n ? dkey[lane] : 0ull;
+          // the candidate list holds the CTA's top keys, and every live token outside
+          // it has a key at or below theta.  A rebuild can leave only mc of them (when
+          // one warp owns the CTA's best mc + 1 keys, its last one is theta itself), so
+          // the bound slot mc takes theta whenever the list is that short.
+          if (lane < kTop) top5[lane] = lane < d_n ? dkey[lane] : (lane == a.mc ? d_theta : 0ull);
         } else {
         constexpr int nk = kSelectWarps * kTop;   // the warps' ranked keys
         constexpr int kPerLane = (nk + 31) / 32;
