@@ -242,10 +242,9 @@ class ClockSampler:
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "select_kernel_traffic.txt")
 
 
-def measured_traffic(kernel_source: str, workload: str):
-    """DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) recorded
-    from an ncu capture of this workload, or None when the kernel source has changed
-    since (its SHA-256 no longer matches the one recorded with the counters).
+def traffic_record(kernel_source: str, workload: str):
+    """The ncu record of this workload: (DRAM bytes per launch, whether the kernel
+    source still has the SHA-256 recorded with the counters), or None.
     The record is `key value` lines; a `workload` line starts each entry."""
     import hashlib
     rec, cur = {}, None
@@ -265,9 +264,17 @@ def measured_traffic(kernel_source: str, workload: str):
     except OSError:
         return None
     r = rec.get(workload)
-    if not r or r.get("source_sha256") != digest or "dram_bytes_per_launch" not in r:
+    if not r or "dram_bytes_per_launch" not in r:
         return None
-    return int(r["dram_bytes_per_launch"])
+    return int(r["dram_bytes_per_launch"]), r.get("source_sha256") == digest
+
+
+def measured_traffic(kernel_source: str, workload: str):
+    """DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) recorded
+    from an ncu capture of this workload, or None when the kernel source has changed
+    since (its SHA-256 no longer matches the one recorded with the counters)."""
+    r = traffic_record(kernel_source, workload)
+    return r[0] if r is not None and r[1] else None
 
 
 def peaks():
@@ -481,6 +488,20 @@ PAPER_CONTEXT = {
 }
 
 
+def earlier_capture(kernel_source, workload, select_ms, hbm):
+    """The ncu DRAM bytes recorded for this workload on an earlier source of the
+    kernel, when the current source has none: reported beside the roofline, never
+    used for its `traffic` or `frac`."""
+    r = traffic_record(kernel_source, workload)
+    if r is None or r[1]:
+        return {}
+    return {"traffic_earlier_source": {
+        "dram_bytes_per_launch": r[0],
+        "frac_at_this_time": r[0] / (select_ms / 1e3) / 1e9 / hbm,
+        "note": "ncu capture of an earlier source of the kernel (the record's SHA-256 no "
+                "longer matches); for context only"}}
+
+
 def selection_roofline(wl, select_ms, hbm, bf16_peak, traffic):
     """Roofline of select_kernel against real resources.  `achieved` is the DRAM
     rate: bytes per launch recorded by ncu for this workload and kernel source
@@ -565,6 +586,7 @@ def measure_config(name, budget, rank, dev, last, seconds, hbm, bf16_peak):
            "select_dram_frac": rl["frac"] if traffic is not None else None,
            "select_compulsory_frac": rl["compulsory_frac"],
            "select_tensor_frac": rl["tensor_frac"], "select_dram_bytes": traffic}
+    out |= earlier_capture("select_impl.cuh", key, se, hbm)
     del q, k, x, w, idx, xs, ws
     torch.cuda.empty_cache()
     return out
@@ -696,7 +718,8 @@ def main():
         "roofline": selection_roofline(wl, select_ms, hbm, bf16_peak,
                                        measured_traffic("select_impl.cuh", key))
                     | {"peak_note": f"{pk_kind} HBM copy bandwidth (of {pk_kind}); tensor peak: "
-                                    f"{pk_kind} cuBLAS bf16 burst"},
+                                    f"{pk_kind} cuBLAS bf16 burst"}
+                    | earlier_capture("select_impl.cuh", key, select_ms, hbm),
         "clocks": clocks,
         "prune_bytes_moved": {"compulsory_bytes": comp, "greedy_feature_bytes": greedy,
                               "compulsory_frac": comp / (total_ms / K / 1e3) / 1e9 / hbm,
