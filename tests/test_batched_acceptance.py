@@ -17,7 +17,9 @@ exactly the sequential greedy's picks in order, for cluster sizes 1-12, publishe
 counts 4-16, lists of 16 and 32 and per-round caps of 16 and 32, on clustered,
 duplicated (exact ties), uniform-weight and video-like features, including k = N.
 It also pins the round counts the design relies on: a longer list never needs
-more rounds on these inputs, and on the video-like request it needs clearly fewer.
+more rounds on these inputs, on the video-like request it needs clearly fewer, and
+on one request of the video batch (16384 tokens, k = 2048, 12 CTAs) the rounds
+fall from about 163 with a 16-entry list to about 100 with a 32-entry one.
 """
 import numpy as np
 import pytest
@@ -144,3 +146,61 @@ def test_longer_list_needs_fewer_rounds():
         assert r32 <= r16, name
         if name == "video":
             assert r32 < 0.8 * r16, (r16, r32)
+
+
+def _rounds_vectorised(xn, w, k, C, mc, lcap, max_accept=32):
+    """The same rounds on unit rows `xn` (float32), with the distance rows computed
+    as they are needed: the round count on a request of the video batch's size."""
+    n = xn.shape[0]
+    bounds = np.linspace(0, n, C + 1).astype(int)
+    sel = np.zeros(n, bool)
+    seed = int(np.argmax(w))
+    sel[seed] = True
+    delta = 1.0 - xn @ xn[seed]
+    taken, rounds = 1, 0
+    idx = np.arange(n)
+    while taken < k:
+        rounds += 1
+        key = np.where(sel, -np.inf, w * delta)
+        pub, U = [], NONE
+        for q in range(C):
+            lo, hi = bounds[q], bounds[q + 1]
+            order = np.lexsort((idx[lo:hi], -key[lo:hi]))      # best first, lowest index on ties
+            top = [int(t) + lo for t in order[:mc + 1] if not sel[int(t) + lo]]
+            pub.extend(_key(key[t], t) for t in top[:mc])
+            U = max(U, _key(key[top[mc]], top[mc]) if len(top) > mc else NONE)
+        above = sorted((c for c in pub if c > U), reverse=True)
+        L = [-c[1] for c in above[:lcap]]
+        Up = max(U, above[lcap]) if len(above) > lcap else U
+        cd = {i: delta[i] for i in L}
+        pending, acc = list(L), []
+        while pending and taken + len(acc) < k and len(acc) < max_accept:
+            b = max(pending, key=lambda i: _key(w[i] * cd[i], i))
+            if not _key(w[b] * cd[b], b) > Up:
+                break
+            acc.append(b)
+            pending.remove(b)
+            for i in pending:
+                cd[i] = min(cd[i], 1.0 - float(xn[i] @ xn[b]))
+        assert acc
+        sel[acc] = True
+        delta = np.minimum(delta, 1.0 - (xn @ xn[acc].T).max(axis=1))
+        taken += len(acc)
+    return rounds
+
+
+def test_video_request_round_counts(oracle_mod):
+    """One request of the video batch (16384 tokens of 2048 features, k = 2048, 12
+    CTAs publishing 16 keys each): about 163 rounds with a 16-entry list and about
+    100 with a 32-entry one, the counts the selection kernel's launcher weighs."""
+    from workloads import config, bf16_bits_to_f32
+    wl = config("c5", budget=12.5, batch=1, seed=4)
+    w = oracle_mod.scores(wl.q, wl.k, wl.cu_seqlens, wl.vis_start, wl.cu_vis,
+                          num_kv_heads=wl.num_kv_heads, scale=wl.scale).astype(np.float32)
+    x = bf16_bits_to_f32(wl.x)
+    xn = (x / np.linalg.norm(x.astype(np.float64), axis=1)[:, None]).astype(np.float32)
+    k = int(wl.cu_keep[1])
+    r16 = _rounds_vectorised(xn, w, k, 12, 16, 16)
+    r32 = _rounds_vectorised(xn, w, k, 12, 16, 32)
+    assert 150 <= r16 <= 175, r16
+    assert r32 <= 0.7 * r16, (r16, r32)
